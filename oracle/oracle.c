@@ -1,0 +1,431 @@
+/*
+ * CPU oracle for the MoE layer forward: MoE Gate -> Fused MoE -> Weight Sum.
+ *
+ * TEST INFRASTRUCTURE. Only the tests, the smoke check and the benchmark's
+ * CPU-baseline leg use this file; the product library never links, loads or
+ * calls it, and it shares no code, header or table with the CUDA path.
+ *
+ * What the paper fixes: the layer's semantic skeleton is the three nodes
+ * MoE Gate, Fused MoE and Weight Sum (Fig. 1 in Section 1; Fig. 3 and its
+ * discussion in Section 5.1), and the
+ * model's mathematical semantics may not change under any implementation
+ * route (Model Semantics Invariant, Section 3.3). It prints no formula for
+ * any node. Each function below therefore writes out the standard definition
+ * of its node in the plainest form, and states the reading it takes where the
+ * paper is silent. Floating point is fp64 except where the result decides an
+ * integer (the expert choice): there the decision is taken in fp32, in a fixed
+ * operation order that the GPU path reproduces, so routing can be compared
+ * bit for bit.
+ *
+ * Compile with -ffp-contract=off: every a*b+c below that is meant as one
+ * rounding is written as fmaf(); everything else must round after each step.
+ */
+#include <math.h>
+#include <pthread.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+/* ----------------------------------------------------------- threading */
+
+typedef void (*range_fn)(void* ctx, int64_t begin, int64_t end);
+typedef struct { range_fn fn; void* ctx; int64_t begin, end; } job_t;
+
+static int g_threads = 1;
+void oracle_set_threads(int n) { g_threads = n < 1 ? 1 : (n > 256 ? 256 : n); }
+int oracle_get_threads(void) { return g_threads; }
+
+static void* job_main(void* p) {
+    job_t* j = (job_t*)p;
+    j->fn(j->ctx, j->begin, j->end);
+    return NULL;
+}
+
+/* Splits [0, n) into contiguous ranges, one per thread. Work items are
+ * independent, so the split never changes a result. */
+static void parallel_for(int64_t n, range_fn fn, void* ctx) {
+    int nt = g_threads;
+    if (nt > n) nt = (int)(n > 0 ? n : 1);
+    if (nt <= 1) { fn(ctx, 0, n); return; }
+    pthread_t th[256];
+    job_t jobs[256];
+    int ok[256];
+    int64_t chunk = (n + nt - 1) / nt;
+    for (int t = 0; t < nt; ++t) {
+        jobs[t].fn = fn; jobs[t].ctx = ctx;
+        jobs[t].begin = t * chunk < n ? t * chunk : n;
+        jobs[t].end = (t + 1) * chunk < n ? (t + 1) * chunk : n;
+        ok[t] = pthread_create(&th[t], NULL, job_main, &jobs[t]) == 0;
+        if (!ok[t]) fn(ctx, jobs[t].begin, jobs[t].end);
+    }
+    for (int t = 0; t < nt; ++t)
+        if (ok[t]) pthread_join(th[t], NULL);
+}
+
+/* ============================================================ MoE Gate */
+
+/*
+ * Router logits l[t,e] = x[t,:] . Wg[e,:] (+ logit_bias[e]), in fp32.
+ *
+ * Reading (the paper gives no order): the dot product is split over 32
+ * partial sums. Partial sum p (p = 0..31) takes the 8-element chunks
+ * c = p, p+32, p+64, ... (chunk c covers elements 8c..8c+7) in increasing c
+ * and, inside a chunk, increasing element, each step one fused multiply-add.
+ * The 32 partial sums are then combined pairwise: at offset d = 16, 8, 4, 2, 1
+ * every partial sum p becomes s[p] + s[p xor d]. Because one addition is
+ * commutative, all 32 end equal, and that value is the logit. The bias is
+ * then added with one fp32 addition. Requires H to be a multiple of 256.
+ */
+typedef struct {
+    int64_t H, E;
+    const float *x, *wg, *bias;
+    float* logits;
+} logit_ctx;
+
+static float pinned_dot(const float* a, const float* b, int64_t H) {
+    float s[32];
+    for (int p = 0; p < 32; ++p) s[p] = 0.0f;
+    for (int64_t c = 0; c < H / 8; ++c) {
+        int p = (int)(c % 32);
+        for (int i = 0; i < 8; ++i) s[p] = fmaf(a[8 * c + i], b[8 * c + i], s[p]);
+    }
+    for (int d = 16; d >= 1; d /= 2) {
+        float n[32];
+        for (int p = 0; p < 32; ++p) n[p] = s[p] + s[p ^ d];
+        for (int p = 0; p < 32; ++p) s[p] = n[p];
+    }
+    return s[0];
+}
+
+static void logit_range(void* vp, int64_t b, int64_t e) {
+    logit_ctx* c = (logit_ctx*)vp;
+    for (int64_t t = b; t < e; ++t)
+        for (int64_t x = 0; x < c->E; ++x) {
+            float l = pinned_dot(c->x + t * c->H, c->wg + x * c->H, c->H);
+            if (c->bias) l = l + c->bias[x];
+            c->logits[t * c->E + x] = l;
+        }
+}
+
+int oracle_gate_logits(int64_t T, int64_t H, int64_t E, const float* x, const float* wg,
+                       const float* logit_bias, float* logits) {
+    if (H % 256 != 0 || T < 0 || E < 1) return -1;
+    logit_ctx c = {H, E, x, wg, logit_bias, logits};
+    parallel_for(T, logit_range, &c);
+    return 0;
+}
+
+/*
+ * Pinned fp32 exponential, used where an exponential decides the expert
+ * choice (sigmoid scores plus a selection bias). Written from the
+ * mathematics, not from any library:
+ *   clamp x to [-86, 88] so that the result stays a normal number;
+ *   n = rint(x * log2(e));  r = (x - n*ln2_hi) - n*ln2_lo  (Cody and Waite,
+ *   "Software Manual for the Elementary Functions", 1980: ln2_hi keeps the
+ *   leading 16 bits of ln 2 so that n*ln2_hi is exact);
+ *   exp(r) by its Taylor series to degree 8, evaluated by Horner's rule with
+ *   a separate multiply and add at each step (|r| <= 0.347, the truncation
+ *   error is below 3e-10 relative);  result = p * 2^n built from exponent
+ *   bits. Every step is one IEEE fp32 operation in this order.
+ */
+static float f32_from_bits(uint32_t u) { float f; memcpy(&f, &u, 4); return f; }
+
+float oracle_pexp(float x) {
+    const float log2e = f32_from_bits(0x3fb8aa3bu);  /* fp32(1/ln 2)           */
+    const float ln2_hi = f32_from_bits(0x3f317200u); /* ln 2, 16 leading bits   */
+    const float ln2_lo = f32_from_bits(0x35bfbe8eu); /* fp32(ln 2 - ln2_hi)     */
+    static const uint32_t inv_fact[9] = {              /* fp32(1/i!), i = 0..8   */
+        0x3f800000u, 0x3f800000u, 0x3f000000u, 0x3e2aaaabu, 0x3d2aaaabu,
+        0x3c088889u, 0x3ab60b61u, 0x39500d01u, 0x37d00d01u};
+    if (x < -86.0f) x = -86.0f;
+    if (x > 88.0f) x = 88.0f;
+    float t = x * log2e;
+    float n = rintf(t);
+    float r = x - n * ln2_hi;
+    r = r - n * ln2_lo;
+    float p = f32_from_bits(inv_fact[8]);
+    for (int i = 7; i >= 0; --i) {
+        p = p * r;
+        p = p + f32_from_bits(inv_fact[i]);
+    }
+    uint32_t bits = (uint32_t)((int32_t)n + 127) << 23;
+    return p * f32_from_bits(bits);
+}
+
+/* Sigmoid score in fp32: s = 1 / (1 + pexp(-l)), IEEE division. */
+float oracle_sigmoid(float l) {
+    float d = 1.0f + oracle_pexp(-l);
+    return 1.0f / d;
+}
+
+typedef struct {
+    int32_t T, E, top_k;
+    int32_t score;       /* 0 = softmax, 1 = sigmoid */
+    int32_t renormalize; /* 1: weights over the selected experts sum to 1 (x scale) */
+    int32_t n_group, topk_group;
+    float routed_scale;
+} oracle_route_cfg;
+
+/* Index of the largest key among those with allowed[e] != 0; the lowest index
+ * wins a tie (the scan is ascending and only a strictly larger key replaces). */
+static int argmax_allowed(const float* key, const unsigned char* allowed, int n) {
+    int best = -1;
+    for (int e = 0; e < n; ++e) {
+        if (!allowed[e]) continue;
+        if (best < 0 || key[e] > key[best]) best = e;
+    }
+    return best;
+}
+
+/*
+ * Expert selection and routing weights for every token.
+ *
+ * Softmax scoring (reading): the selection key is the logit itself (softmax
+ * is increasing, so ordering by logit equals ordering by probability and no
+ * exponential decides the choice). The top_k largest keys are taken in
+ * descending order, equal keys going to the lower expert index. Weights, in
+ * fp64: renormalised, w_j = exp(l_j - m) / sum over selected exp(l_i - m) with
+ * m the largest selected logit; otherwise the full softmax over all E experts
+ * evaluated at the selected ones. Both are multiplied by routed_scale.
+ *
+ * Sigmoid scoring with group-limited selection (reading, following the
+ * DeepSeek-V3 description of this router): s_e = sigmoid(l_e) in fp32
+ * (pinned exponential), q_e = s_e + select_bias[e] (fp32, bias used for the
+ * choice only). Experts form n_group contiguous groups; a group's score is
+ * the fp32 sum of its two largest q. The topk_group best groups are kept
+ * (ties to the lower group), then the top_k largest q inside kept groups are
+ * taken in descending order (ties to the lower expert). Weights, in fp64:
+ * w_j = s_j / sum over selected s (renormalised) or s_j, times routed_scale.
+ * With n_group = 1 the group step keeps every expert.
+ *
+ * ids[t*top_k + j] is the j-th selected expert, w[t*top_k + j] its weight.
+ */
+int oracle_route(const oracle_route_cfg* c, const float* logits, const float* select_bias,
+                 int32_t* ids, double* w) {
+    const int E = c->E, k = c->top_k;
+    if (k < 1 || k > E) return -1;
+    if (c->score == 1) {
+        if (c->n_group < 1 || E % c->n_group) return -1;
+        if (c->n_group > 1 && E / c->n_group < 2) return -1;
+        if (c->topk_group < 1 || c->topk_group > c->n_group) return -1;
+        if (k > c->topk_group * (E / c->n_group)) return -1;
+    }
+    float* key = (float*)malloc(sizeof(float) * E);
+    float* s = (float*)malloc(sizeof(float) * E);
+    unsigned char* allowed = (unsigned char*)malloc(E);
+    const int G = c->n_group > 0 ? c->n_group : 1;
+    float* gscore = (float*)malloc(sizeof(float) * G);
+    unsigned char* gallowed = (unsigned char*)malloc(G);
+    for (int64_t t = 0; t < c->T; ++t) {
+        const float* l = logits + t * E;
+        int32_t* id = ids + t * k;
+        double* wt = w + t * k;
+        if (c->score == 0) {
+            for (int e = 0; e < E; ++e) { key[e] = l[e]; allowed[e] = 1; }
+        } else {
+            for (int e = 0; e < E; ++e) {
+                s[e] = oracle_sigmoid(l[e]);
+                key[e] = select_bias ? s[e] + select_bias[e] : s[e];
+                allowed[e] = 1;
+            }
+            if (G > 1) {
+                const int gs = E / G;
+                for (int g = 0; g < G; ++g) {
+                    /* the two largest q of group g */
+                    int a = -1, b = -1;
+                    for (int e = g * gs; e < (g + 1) * gs; ++e) {
+                        if (a < 0 || key[e] > key[a]) { b = a; a = e; }
+                        else if (b < 0 || key[e] > key[b]) b = e;
+                    }
+                    gscore[g] = key[a] + key[b];
+                    gallowed[g] = 1;
+                }
+                unsigned char* kept = (unsigned char*)calloc(G, 1);
+                for (int r = 0; r < c->topk_group; ++r) {
+                    int g = argmax_allowed(gscore, gallowed, G);
+                    kept[g] = 1;
+                    gallowed[g] = 0;
+                }
+                for (int e = 0; e < E; ++e) allowed[e] = kept[e / gs];
+                free(kept);
+            }
+        }
+        for (int j = 0; j < k; ++j) {
+            int e = argmax_allowed(key, allowed, E);
+            id[j] = e;
+            allowed[e] = 0;
+        }
+        if (c->score == 0) {
+            if (c->renormalize) {
+                double m = (double)l[id[0]], z = 0.0;
+                for (int j = 0; j < k; ++j) z += exp((double)l[id[j]] - m);
+                for (int j = 0; j < k; ++j) wt[j] = exp((double)l[id[j]] - m) / z * c->routed_scale;
+            } else {
+                double m = (double)l[0], z = 0.0;
+                for (int e = 1; e < E; ++e) if ((double)l[e] > m) m = (double)l[e];
+                for (int e = 0; e < E; ++e) z += exp((double)l[e] - m);
+                for (int j = 0; j < k; ++j) wt[j] = exp((double)l[id[j]] - m) / z * c->routed_scale;
+            }
+        } else {
+            double z = 0.0;
+            for (int j = 0; j < k; ++j) z += (double)s[id[j]];
+            for (int j = 0; j < k; ++j)
+                wt[j] = (c->renormalize ? (double)s[id[j]] / z : (double)s[id[j]]) * c->routed_scale;
+        }
+    }
+    free(key); free(s); free(allowed); free(gscore); free(gallowed);
+    return 0;
+}
+
+/* ============================================ Fused MoE: permutation */
+
+/*
+ * Groups the P = T*top_k (token, slot) pairs by expert. Pair p = t*top_k + j
+ * goes to expert ids[p]. Reading (order unstated in the paper): a stable
+ * counting sort, experts ascending and pairs ascending inside an expert.
+ *   counts[e]      number of pairs routed to e
+ *   offsets[e]     sum of counts[0..e-1] (offsets[E] = P)
+ *   sorted_pair[r] the pair at sorted position r
+ *   pair_pos[p]    the sorted position of pair p (inverse of sorted_pair)
+ */
+int oracle_permute(int64_t P, int32_t E, const int32_t* ids, int32_t* counts, int32_t* offsets,
+                   int32_t* sorted_pair, int32_t* pair_pos) {
+    for (int e = 0; e < E; ++e) counts[e] = 0;
+    for (int64_t p = 0; p < P; ++p) {
+        if (ids[p] < 0 || ids[p] >= E) return -1;
+        counts[ids[p]] += 1;
+    }
+    offsets[0] = 0;
+    for (int e = 0; e < E; ++e) offsets[e + 1] = offsets[e] + counts[e];
+    int64_t r = 0;
+    for (int e = 0; e < E; ++e)
+        for (int64_t p = 0; p < P; ++p)
+            if (ids[p] == e) {
+                sorted_pair[r] = (int32_t)p;
+                pair_pos[p] = (int32_t)r;
+                ++r;
+            }
+    return 0;
+}
+
+/* ============================== Fused MoE: stored weight formats */
+
+/*
+ * FP8 E4M3 value of a byte (the OCP 8-bit floating point format, "fn"
+ * variant): sign bit, 4 exponent bits with bias 7, 3 mantissa bits;
+ * exponent field 0 gives subnormals m * 2^-9; no infinities; S.1111.111 is
+ * NaN. Block-wise E4M3 expert weights are the format named in Section 6.2.
+ */
+double oracle_e4m3_value(uint8_t code) {
+    int sign = code >> 7, ex = (code >> 3) & 0xf, m = code & 7;
+    double v;
+    if (ex == 15 && m == 7) return NAN;
+    if (ex == 0) v = ldexp((double)m, -9);
+    else v = ldexp(1.0 + m / 8.0, ex - 7);
+    return sign ? -v : v;
+}
+
+/* Dequantised weight of one [N, K] expert matrix stored as e4m3 codes with
+ * one fp32 scale per 128x128 block: W[n,k] = e4m3(q[n,k]) * s[n/128][k/128],
+ * exact in fp64. */
+void oracle_dequant_fp8_b128(int64_t N, int64_t K, const uint8_t* q, const float* s, double* out) {
+    for (int64_t n = 0; n < N; ++n)
+        for (int64_t k = 0; k < K; ++k)
+            out[n * K + k] = oracle_e4m3_value(q[n * K + k]) * (double)s[(n / 128) * (K / 128) + k / 128];
+}
+
+static double bf16_value(uint16_t h) { return (double)f32_from_bits((uint32_t)h << 16); }
+
+/* Dequantised weight of one [N, K] expert matrix stored as symmetric int4
+ * (two's complement nibble, element 2i in the low nibble of byte i of a row)
+ * with one bf16 scale per 128 consecutive k: W[n,k] = q[n,k] * s[n][k/128],
+ * exact in fp64. */
+void oracle_dequant_int4_g128(int64_t N, int64_t K, const uint8_t* q, const uint16_t* s, double* out) {
+    for (int64_t n = 0; n < N; ++n)
+        for (int64_t k = 0; k < K; ++k) {
+            uint8_t byte = q[n * (K / 2) + k / 2];
+            int v = (k % 2 == 0) ? (byte & 0xf) : (byte >> 4);
+            if (v >= 8) v -= 16;
+            out[n * K + k] = (double)v * bf16_value(s[n * (K / 128) + k / 128]);
+        }
+}
+
+void oracle_pexp_n(int64_t n, const float* in, float* out) {
+    for (int64_t i = 0; i < n; ++i) out[i] = oracle_pexp(in[i]);
+}
+
+void oracle_sigmoid_n(int64_t n, const float* in, float* out) {
+    for (int64_t i = 0; i < n; ++i) out[i] = oracle_sigmoid(in[i]);
+}
+
+void oracle_widen_f32(int64_t n, const float* in, double* out) {
+    for (int64_t i = 0; i < n; ++i) out[i] = (double)in[i];
+}
+
+void oracle_widen_bf16(int64_t n, const uint16_t* in, double* out) {
+    for (int64_t i = 0; i < n; ++i) out[i] = bf16_value(in[i]);
+}
+
+/* ============================== Fused MoE: one expert's SwiGLU FFN */
+
+/*
+ * For each of n_rows activation rows x (fp64, length H) routed to one expert:
+ *   g = Wgate x,  u = Wup x            (Wgate, Wup: [I, H])
+ *   a_i = silu(g_i) * u_i,  silu(z) = z / (1 + exp(-z))
+ *   y = Wdown a                        (Wdown: [H, I])
+ * all in fp64. The expert FFN is the standard gated (SwiGLU) MLP of the
+ * MoE models the paper serves (Section 6); the paper does not print it.
+ */
+typedef struct {
+    int64_t H, I;
+    const double *x, *wg, *wu, *wd;
+    double* y;
+} ffn_ctx;
+
+static void ffn_range(void* vp, int64_t b, int64_t e) {
+    ffn_ctx* c = (ffn_ctx*)vp;
+    double* a = (double*)malloc(sizeof(double) * c->I);
+    for (int64_t r = b; r < e; ++r) {
+        const double* x = c->x + r * c->H;
+        for (int64_t i = 0; i < c->I; ++i) {
+            double g = 0.0, u = 0.0;
+            for (int64_t h = 0; h < c->H; ++h) {
+                g += c->wg[i * c->H + h] * x[h];
+                u += c->wu[i * c->H + h] * x[h];
+            }
+            a[i] = g / (1.0 + exp(-g)) * u;
+        }
+        double* y = c->y + r * c->H;
+        for (int64_t n = 0; n < c->H; ++n) {
+            double acc = 0.0;
+            for (int64_t i = 0; i < c->I; ++i) acc += c->wd[n * c->I + i] * a[i];
+            y[n] = acc;
+        }
+    }
+    free(a);
+}
+
+void oracle_expert_ffn(int64_t n_rows, int64_t H, int64_t I, const double* x, const double* w_gate,
+                       const double* w_up, const double* w_down, double* y) {
+    ffn_ctx c = {H, I, x, w_gate, w_up, w_down, y};
+    parallel_for(n_rows, ffn_range, &c);
+}
+
+/* ==================================================== Weight Sum */
+
+/*
+ * out[t,:] = sum over j of w[t,j] * y_pairs[pair_pos[t*k + j], :]
+ *            (+ y_shared[t,:] when a shared expert is present, weight 1),
+ * in fp64. y_pairs holds one expert output row per sorted pair position.
+ */
+void oracle_combine(int64_t T, int64_t k, int64_t H, const double* y_pairs, const double* w,
+                    const int32_t* pair_pos, const double* y_shared, double* out) {
+    for (int64_t t = 0; t < T; ++t)
+        for (int64_t h = 0; h < H; ++h) {
+            double acc = 0.0;
+            for (int64_t j = 0; j < k; ++j)
+                acc += w[t * k + j] * y_pairs[(int64_t)pair_pos[t * k + j] * H + h];
+            if (y_shared) acc += y_shared[t * H + h];
+            out[t * H + h] = acc;
+        }
+}
