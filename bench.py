@@ -1,0 +1,364 @@
+#!/usr/bin/env python
+"""MoE layer forward throughput on GB300 (tokens/s), one JSON line.
+
+  python bench.py [--gpus N --steps K --warmup W] [--impl ours|reference] [--workload ID]
+
+A step is one full layer forward (MoE Gate, permutation, expert FFNs,
+Weight Sum) over one batch of the workload, through the C ABI (moe_forward)
+on inputs already resident in HBM. The default workload is the decode-shaped
+bf16 layer: T=32 tokens, hidden 4096, 128 experts, top-8, intermediate 1536.
+Its active experts' weights (~4.2 GB) exceed the 126 MB L2, so no flush is
+needed between steps. With N GPUs (torchrun) every rank runs its own replica
+on its own batch (the layer has no exchange step here): weak scaling.
+
+--impl reference times the CPU oracle (test infrastructure, plain C) on the
+host cores on a bounded token sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import ctypes
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+METRIC = "MoE layer tokens/sec at 1 GB300; % of HBM (decode) / tensor-core (prefill) roofline"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    return FALLBACK_PEAKS, "fallback"
+
+
+# ------------------------------------------------------------------ clocks
+
+class ClockSampler:
+    """Samples SM clock and clock-event reasons of this process's GPU during
+    the timed region (NVML through ctypes; nvidia-smi if NVML is missing)."""
+
+    REASONS = {0x1: "gpu_idle", 0x2: "applications_clocks_setting", 0x4: "sw_power_cap", 0x8: "hw_slowdown",
+               0x10: "sync_boost", 0x20: "sw_thermal_slowdown", 0x40: "hw_thermal_slowdown",
+               0x80: "hw_power_brake_slowdown", 0x100: "display_clock_setting"}
+
+    def __init__(self, uuid: str | None, period_s: float = 0.002):
+        self.uuid, self.period = uuid, period_s
+        self.samples, self.reasons = [], 0
+        self.max_mhz = None
+        self._stop = threading.Event()
+        self._nvml = None
+        self._h = None
+        try:
+            nv = ctypes.CDLL("libnvidia-ml.so.1")
+            if nv.nvmlInit_v2() == 0:
+                h = ctypes.c_void_p()
+                if uuid and nv.nvmlDeviceGetHandleByUUID(uuid.encode(), ctypes.byref(h)) == 0:
+                    self._nvml, self._h = nv, h
+                    m = ctypes.c_uint()
+                    if nv.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(m)) == 0:
+                        self.max_mhz = m.value
+        except OSError:
+            self._nvml = None
+
+    def _run(self):
+        nv, h = self._nvml, self._h
+        clk, rs = ctypes.c_uint(), ctypes.c_ulonglong()
+        fn = getattr(nv, "nvmlDeviceGetCurrentClocksEventReasons", None) or nv.nvmlDeviceGetCurrentClocksThrottleReasons
+        while not self._stop.is_set():
+            if nv.nvmlDeviceGetClockInfo(h, 1, ctypes.byref(clk)) == 0:
+                self.samples.append(clk.value)
+            if fn(h, ctypes.byref(rs)) == 0:
+                self.reasons |= rs.value
+            time.sleep(self.period)
+
+    def __enter__(self):
+        if self._nvml is not None:
+            self._t = threading.Thread(target=self._run, daemon=True)
+            self._t.start()
+        else:
+            self._proc = subprocess.Popen(
+                ["nvidia-smi", "--query-gpu=clocks.sm,clocks.max.sm,clocks_event_reasons.active", "--format=csv,noheader,nounits",
+                 "-lms", "100"] + ([f"--id={self.uuid}"] if self.uuid else []),
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        return self
+
+    def __exit__(self, *a):
+        if self._nvml is not None:
+            self._stop.set()
+            self._t.join()
+        else:
+            self._proc.terminate()
+            out, _ = self._proc.communicate(timeout=10)
+            for line in out.strip().splitlines():
+                try:
+                    sm, mx, rs = [v.strip() for v in line.split(",")]
+                    self.samples.append(int(sm))
+                    self.max_mhz = int(mx)
+                    self.reasons |= int(rs, 16)
+                except ValueError:
+                    pass
+
+    def summary(self):
+        reasons = [n for b, n in self.REASONS.items() if self.reasons & b and n != "gpu_idle"]
+        return {"sm_mhz": statistics.median(self.samples) if self.samples else None, "sm_max_mhz": self.max_mhz,
+                "reasons": reasons, "samples": len(self.samples)}
+
+
+# --------------------------------------------------------------- workload
+
+def load_workload(wid: int):
+    wl = synth.WORKLOADS[wid]
+    inp = synth.make_inputs(wl)
+    return wl, inp
+
+
+def algorithmic_weight_bytes(wl, active: int) -> int:
+    """Expert weight bytes one layer forward must read: every active expert's
+    three matrices (+ scales), plus the shared expert."""
+    per = 3 * wl.H * wl.I
+    if wl.wq == "bf16":
+        b = per * 2
+    elif wl.wq == "f32":
+        b = per * 4
+    elif wl.wq == "fp8_b128":
+        b = per + 3 * (wl.H // 128) * (wl.I // 128) * 4
+    else:
+        b = per // 2 + 3 * (wl.H * wl.I // 128) * 2
+    total = active * b
+    if wl.has_shared:
+        ps = 3 * wl.H * wl.I_shared
+        total += (ps + 3 * (wl.H // 128) * (wl.I_shared // 128) * 4) if wl.wq == "fp8_b128" else ps * 2
+    return total
+
+
+def cpu_sample_rows(wl, n_tokens: int, step: int) -> list:
+    return [(step * n_tokens + i) % wl.T for i in range(n_tokens)]
+
+
+def run_reference(args, wl, inp, rank):
+    """The oracle on the host cores, a bounded token sample per step."""
+    import oracle
+
+    if rank != 0:
+        return None
+    n_tok = args.ref_tokens
+    for s in range(args.warmup):
+        oracle.forward(wl, inp, rows=cpu_sample_rows(wl, n_tok, s))
+    t0 = time.perf_counter()
+    for s in range(args.steps):
+        oracle.forward(wl, inp, rows=cpu_sample_rows(wl, n_tok, s))
+    dt = time.perf_counter() - t0
+    v = n_tok * args.steps / dt
+    sample = (f"{n_tok} token(s) per step (expert FFNs of those tokens; router logits, expert choice and "
+              f"permutation for all {wl.T} tokens), fp64 C oracle")
+    return {"metric": METRIC, "impl": "reference", "value": v, "unit": "tokens/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": workload_config(wl),
+            "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": oracle.get_threads(), "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def workload_config(wl):
+    return {"workload": wl.name, "T": wl.T, "H": wl.H, "I": wl.I, "E": wl.E, "top_k": wl.top_k,
+            "scoring": wl.score, "activations": wl.act, "weights": wl.wq,
+            "shared_expert": bool(wl.has_shared), "parallelism": "replicas",
+            "l2": "no flush: the active experts' weights read each step exceed the 126 MB L2"}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", type=int, default=2, help="synth.WORKLOADS id (2 = decode bf16)")
+    ap.add_argument("--route", default="auto", choices=["auto", "stream", "simt", "tc"])
+    ap.add_argument("--ref-tokens", type=int, default=1, help="tokens per oracle step (reference arm)")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "ours":
+        args.warmup = 3
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        wl, inp = load_workload(args.workload)
+        print(json.dumps(run_reference(args, wl, inp, rank)))
+        return
+
+    import torch
+
+    import paper_2607_12875_gb300 as gb
+
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+
+    wl, inp = load_workload(args.workload)
+    dev = torch.device("cuda", local)
+
+    def act(a):
+        if wl.act == "f32":
+            return torch.from_numpy(a).to(dev)
+        return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).to(dev).view(torch.bfloat16)
+
+    def wts(store):
+        d = {}
+        for k, v in store.items():
+            d[k] = torch.from_numpy(v.view(np.int16) if v.dtype == np.uint16 else v).to(dev)
+        return gb.weights(d["w_gate"], d["w_up"], d["w_down"], d.get("s_gate"), d.get("s_up"), d.get("s_down")), d
+
+    x = act(inp["x"])
+    wr = act(inp["w_router"])
+    lb = None if inp["logit_bias"] is None else torch.from_numpy(inp["logit_bias"]).to(dev)
+    sb = None if inp["select_bias"] is None else torch.from_numpy(inp["select_bias"]).to(dev)
+    experts, keep1 = wts(inp["experts"])
+    shared, keep2 = wts(inp["shared"]) if wl.has_shared else (None, None)
+    cfg = gb.make_config(wl.T, wl.H, wl.I, wl.E, wl.top_k, score=wl.score, renormalize=wl.renormalize,
+                         n_group=wl.n_group, topk_group=wl.topk_group, routed_scale=wl.routed_scale, act=wl.act,
+                         w=wl.wq, has_shared=wl.has_shared, I_shared=wl.I_shared, ffn_route=args.route)
+    ws = torch.empty(gb.workspace_size(cfg), dtype=torch.uint8, device=dev)
+    out = torch.empty((wl.T, wl.H), dtype=x.dtype, device=dev)
+    counts = torch.empty(wl.E, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        gb.moe_forward(cfg, x, wr, lb, sb, experts, shared, out, ws)
+
+    for _ in range(args.warmup):
+        step()
+    gb.moe_forward(cfg, x, wr, lb, sb, experts, shared, out, ws, counts=counts)
+    torch.cuda.synchronize()
+    if gb.moe_device_status(ws) != gb.OK:
+        raise RuntimeError("device-side wait timed out during warm-up")
+    active = int((counts.cpu() > 0).sum())
+
+    uuid = None
+    try:
+        uuid = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid)
+    except Exception:
+        pass
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(uuid) as clocks:
+        start.record(stream)
+        for _ in range(args.steps):
+            step()
+        end.record(stream)
+        torch.cuda.synchronize()
+    barrier()
+    ms = start.elapsed_time(end)
+    if dist is not None:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    value = wl.T * args.steps * world / (ms / 1e3)
+
+    # dominant kernel: the expert FFN, timed through its own entry point on the same stream
+    P = wl.P
+    ids = torch.empty((wl.T, wl.top_k), dtype=torch.int32, device=dev)
+    w = torch.empty((wl.T, wl.top_k), dtype=torch.float32, device=dev)
+    offs = torch.empty(wl.E + 1, dtype=torch.int32, device=dev)
+    sp = torch.empty(P, dtype=torch.int32, device=dev)
+    pp = torch.empty(P, dtype=torch.int32, device=dev)
+    y = torch.empty((P, wl.H), dtype=x.dtype, device=dev)
+    gb.moe_route(cfg, x, wr, lb, sb, ids, w, ws)
+    gb.moe_permute(cfg, ids, counts, offs, sp, pp, ws)
+    for _ in range(3):
+        gb.moe_grouped_ffn(cfg, x, counts, offs, sp, experts, y, ws)
+    fs, fe = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    fs.record(stream)
+    for _ in range(args.steps):
+        gb.moe_grouped_ffn(cfg, x, counts, offs, sp, experts, y, ws)
+    fe.record(stream)
+    torch.cuda.synchronize()
+    ffn_ms = fs.elapsed_time(fe) / args.steps
+    pk, pk_kind = peaks()
+    routed_bytes = algorithmic_weight_bytes(wl.replace(has_shared=False), active)
+    achieved = routed_bytes / (ffn_ms / 1e3) / 1e9
+    roofline = {"bound": "hbm", "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s",
+                "frac": achieved / pk["hbm_gbs"], "traffic": None, "peak_kind": pk_kind,
+                "kernel": "moe_grouped_ffn (weight-streaming route: gate/up + down)",
+                "algorithmic_bytes": routed_bytes, "active_experts": active, "ms_per_launch": ffn_ms}
+
+    # end to end through the public host-buffer entry point
+    x_host = x.cpu().pin_memory()
+    out_host = torch.empty((wl.T, wl.H), dtype=x.dtype).pin_memory()
+    for _ in range(3):
+        gb.moe_forward_hostio(cfg, x_host, wr, lb, sb, experts, shared, out_host, ws)
+    torch.cuda.synchronize()
+    barrier()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        gb.moe_forward_hostio(cfg, x_host, wr, lb, sb, experts, shared, out_host, ws)
+        stream.synchronize()
+    e2e_s = time.perf_counter() - t0
+    barrier()
+    if dist is not None:
+        t = torch.tensor([e2e_s], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_s = float(t.item())
+    io_bytes = wl.T * wl.H * x.element_size()
+    e2e = {"value": wl.T * args.steps * world / e2e_s, "unit": "tokens/s", "h2d_bytes_per_step": io_bytes,
+           "d2h_bytes_per_step": io_bytes}
+
+    # kernels this library launched per step: gate logits + expert choice, 3 for the
+    # permutation, schedule + 2 per expert-FFN problem, combine
+    per_step = 2 + 3 + 3 + (3 if wl.has_shared else 0) + 1
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+
+        n_tok = min(wl.T, 32)
+        t0 = time.perf_counter()
+        oracle.forward(wl, inp, rows=list(range(n_tok)))
+        dt = time.perf_counter() - t0
+        cpu = {"value": n_tok / dt, "unit": "tokens/s", "cores": oracle.get_threads(), "kind": "oracle",
+               "sample": f"first {n_tok} tokens: full routing of all {wl.T} tokens plus the expert FFNs and "
+                         f"combine of the sampled ones ({dt:.1f} s)"}
+
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+                "vs_baseline": None, "dtype": wl.act if wl.wq in ("f32", "bf16") else f"{wl.act}+{wl.wq}",
+                "data": "synthetic (seeded SplitMix64/Irwin-Hall normals; random-init weights)",
+                "config": workload_config(wl), "clocks": clocks.summary(), "e2e": e2e,
+                "gpu_launches": per_step * args.steps, "roofline": roofline, "cpu_baseline": cpu}
+        print(json.dumps(line))
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,218 @@
+/*
+ * gbmoe.h - C ABI of the GB300 (sm_103a) MoE layer forward.
+ *
+ * The layer is the paper's three-node MoE skeleton (Fig. 1, Section 1;
+ * Fig. 3 and its discussion, Section 5.1):
+ *   MoE Gate    router logits, top-k expert choice and routing weights
+ *               -> moe_route
+ *   Fused MoE   grouping of (token, slot) pairs by expert, then each expert's
+ *               SwiGLU FFN on its rows, with bf16, fp8 (block-scaled E4M3,
+ *               the format named in Section 6.2) or int4 weights
+ *               -> moe_permute, moe_grouped_ffn, moe_shared_ffn
+ *   Weight Sum  routing-weighted sum of each token's expert outputs
+ *               -> moe_combine
+ *   the whole layer -> moe_forward (device buffers) and moe_forward_hostio
+ *   (host activations in and out).
+ * The paper prints no formula for these nodes; the definitions stated below
+ * are the standard ones, and the library reproduces an independent CPU
+ * oracle of them (routing bit for bit, outputs within a per-dtype tolerance).
+ *
+ * Conventions for every call
+ *  - Pointers are DEVICE pointers owned by the caller unless a parameter says
+ *    host. Every tensor is dense, row-major, 16-byte aligned. The library
+ *    never allocates, frees or synchronises (moe_device_status excepted);
+ *    calls are asynchronous on `stream` (a cudaStream_t; NULL = the legacy
+ *    default stream) and run on the current device.
+ *  - Argument errors are found on the host before anything is launched and
+ *    return a negative status; nothing is written then.
+ *  - Calls that take a workspace use it for scratch only; its size comes from
+ *    gbmoe_workspace_size for the same config. Calls sharing one workspace
+ *    must not overlap in time (same stream, or ordered by events).
+ *  - Names: T tokens, H hidden size, E routed experts, k = top_k, I expert
+ *    intermediate size, P = T*k (token, slot) pairs, pair p = t*k + j.
+ */
+#ifndef GBMOE_H
+#define GBMOE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Status codes. */
+enum {
+    GBMOE_OK = 0,
+    GBMOE_EINVAL = -1,          /* null/misaligned pointer, inconsistent config */
+    GBMOE_EUNSUPPORTED = -2,    /* valid config outside what the kernels cover  */
+    GBMOE_EWORKSPACE = -3,      /* workspace smaller than gbmoe_workspace_size  */
+    GBMOE_ECUDA = -4,           /* a CUDA launch or copy failed                 */
+    GBMOE_EDEVICE_TIMEOUT = -5  /* a bounded device-side wait gave up           */
+};
+
+/* Element types. act_dtype uses F32 or BF16; w_dtype any of the four. */
+enum {
+    GBMOE_F32 = 0,
+    GBMOE_BF16 = 1,
+    GBMOE_FP8_E4M3_B128 = 2, /* e4m3 codes + fp32 scale per 128x128 block      */
+    GBMOE_INT4_G128 = 3      /* packed int4 + bf16 scale per 128 along K (row) */
+};
+
+/* Router scoring. */
+enum { GBMOE_SOFTMAX = 0, GBMOE_SIGMOID = 1 };
+
+/* Which expert-FFN kernels run. AUTO streams weights when the average number
+ * of rows per expert P/E is at most 16 and otherwise runs the grouped GEMM
+ * (tensor cores for bf16 activations, CUDA cores for fp32). */
+enum {
+    GBMOE_FFN_AUTO = 0,
+    GBMOE_FFN_STREAM = 1, /* weight streaming: few rows per expert (decode)       */
+    GBMOE_FFN_SIMT = 2,   /* CUDA-core tiled GEMM (fp32 activations, any weights) */
+    GBMOE_FFN_TC = 3      /* tcgen05/TMEM/TMA grouped GEMM (bf16 activations)     */
+};
+
+typedef struct gbmoe_config {
+    int32_t T, H, I, E, top_k;
+    int32_t score;        /* GBMOE_SOFTMAX or GBMOE_SIGMOID                         */
+    int32_t renormalize;  /* 1: the selected experts' weights sum to routed_scale   */
+    int32_t n_group;      /* sigmoid only: E experts in n_group contiguous groups   */
+    int32_t topk_group;   /* sigmoid only: groups kept before the expert choice     */
+    float routed_scale;   /* multiplies every routing weight (1.0 = none)           */
+    int32_t act_dtype;    /* x, router weight, intermediates, out: F32 or BF16      */
+    int32_t w_dtype;      /* routed and shared expert weights                       */
+    int32_t has_shared;   /* 1: add one always-on expert with weight 1              */
+    int32_t I_shared;     /* its intermediate size                                  */
+    int32_t ffn_route;    /* GBMOE_FFN_*                                            */
+} gbmoe_config;
+
+/* One set of expert weights (all experts stacked, E of them, or 1 for the
+ * shared expert). nn.Linear layout: gate and up are [E, I, H], down is
+ * [E, H, I] (output rows, input contiguous).
+ *  F32 / BF16:      w_* hold the values; s_* are NULL.
+ *  FP8_E4M3_B128:   w_* hold e4m3 bytes in the same shape; s_gate, s_up are
+ *                   fp32 [E, I/128, H/128] and s_down fp32 [E, H/128, I/128];
+ *                   W[n,k] = e4m3(q[n,k]) * s[n/128][k/128].
+ *  INT4_G128:       w_* hold packed nibbles, [E, N, K/2] bytes for an [N, K]
+ *                   matrix, element 2i in the low nibble of byte i, two's
+ *                   complement; s_* are bf16 [E, N, K/128];
+ *                   W[n,k] = q[n,k] * s[n][k/128]. */
+typedef struct gbmoe_expert_weights {
+    const void *w_gate, *w_up, *w_down;
+    const void *s_gate, *s_up, *s_down;
+} gbmoe_expert_weights;
+
+/* Human-readable name of a status code (static string). */
+const char* gbmoe_status_string(int status);
+
+/* GBMOE_OK if the config is valid and covered, else the status a call with it
+ * would return. Limits: H % 256 == 0, I % 128 == 0 (I_shared too),
+ * 1 <= E <= 512, 1 <= top_k <= min(E, 32), T >= 0, P <= 2^30. */
+int gbmoe_check_config(const gbmoe_config* cfg);
+
+/* Workspace bytes that moe_forward / moe_forward_hostio need for cfg (the
+ * other calls need no more). 0 if the config is invalid. */
+size_t gbmoe_workspace_size(const gbmoe_config* cfg);
+
+/*
+ * MoE Gate (Fig. 1 and Fig. 3). For every token t:
+ *   l[t,e] = x[t,:] . w_router[e,:] (+ logit_bias[e]), fp32, in a fixed order:
+ *     32 partial sums, partial p takes the 8-element chunks p, p+32, ... in
+ *     order with one fused multiply-add per element, then pairwise sums
+ *     s[p] + s[p xor d] for d = 16, 8, 4, 2, 1, then one fp32 add of the bias;
+ *   softmax: top_k largest l (ties to the lower expert) in descending order;
+ *     weight = exp(l_j - max) / sum over the selected (renormalize) or over
+ *     all E (otherwise), times routed_scale;
+ *   sigmoid: s_e = 1/(1 + exp(-l_e)) with a fixed fp32 exponential,
+ *     q_e = s_e + select_bias[e]; keep the topk_group groups whose two
+ *     largest q sum highest (ties to the lower group), then the top_k largest
+ *     q in kept groups (ties to the lower expert); weight = s_j / sum of
+ *     selected s (renormalize) or s_j, times routed_scale.
+ * x [T, H] and w_router [E, H] are act_dtype. logit_bias [E] fp32 or NULL
+ * (enters the logit, so weights too); select_bias [E] fp32 or NULL (sigmoid
+ * selection only). Writes topk_ids [T, k] int32 and topk_w [T, k] fp32.
+ * Workspace: the logits (T*E fp32).
+ */
+int moe_route(const gbmoe_config* cfg, const void* x, const void* w_router, const float* logit_bias,
+              const float* select_bias, int32_t* topk_ids, float* topk_w, void* workspace,
+              size_t workspace_bytes, void* stream);
+
+/*
+ * Fused MoE, grouping step: stable counting sort of the P pairs by expert.
+ * topk_ids [T, k] int32 (each in [0, E); out-of-range ids are not checked on
+ * the device and give undefined grouping). Writes counts [E], offsets [E+1]
+ * (exclusive prefix sum, offsets[E] = P), sorted_pair [P] (pairs ordered by
+ * expert, then by pair index) and pair_pos [P] (inverse: position of pair p),
+ * all int32. Bit-exact and deterministic.
+ */
+int moe_permute(const gbmoe_config* cfg, const int32_t* topk_ids, int32_t* counts, int32_t* offsets,
+                int32_t* sorted_pair, int32_t* pair_pos, void* workspace, size_t workspace_bytes,
+                void* stream);
+
+/*
+ * Fused MoE, expert FFNs. For every sorted position r of expert e
+ * (offsets[e] <= r < offsets[e+1]) with token t = sorted_pair[r] / k:
+ *   g = Wgate_e x_t, u = Wup_e x_t, a = silu(g) * u, y_pairs[r] = Wdown_e a.
+ * fp32 accumulation; a (the intermediate) and y_pairs are stored in
+ * act_dtype. No routing weight is applied here. x [T, H] act_dtype; counts,
+ * offsets, sorted_pair as produced by moe_permute; y_pairs [P, H] act_dtype.
+ */
+int moe_grouped_ffn(const gbmoe_config* cfg, const void* x, const int32_t* counts, const int32_t* offsets,
+                    const int32_t* sorted_pair, const gbmoe_expert_weights* experts, void* y_pairs,
+                    void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * Shared expert: y_shared[t] = SwiGLU FFN of x_t with the single expert
+ * `shared` (intermediate size I_shared, same w_dtype), for every token.
+ * y_shared [T, H] act_dtype. Requires cfg->has_shared.
+ */
+int moe_shared_ffn(const gbmoe_config* cfg, const void* x, const gbmoe_expert_weights* shared,
+                   void* y_shared, void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * Weight Sum (Fig. 1 and Fig. 3):
+ *   out[t] = sum_{j=0..k-1} topk_w[t,j] * y_pairs[pair_pos[t*k + j]]
+ *            (+ y_shared[t] if y_shared is not NULL),
+ * summed in fp32 in that order and rounded once to act_dtype. A gather per
+ * token: no atomics, deterministic. y_pairs [P, H], y_shared [T, H] or NULL,
+ * out [T, H], all act_dtype; topk_w [T, k] fp32; pair_pos [P] int32.
+ */
+int moe_combine(const gbmoe_config* cfg, const void* y_pairs, const float* topk_w, const int32_t* pair_pos,
+                const void* y_shared, void* out, void* stream);
+
+/*
+ * The whole layer: moe_route, moe_permute, moe_grouped_ffn, moe_shared_ffn
+ * (if cfg->has_shared) and moe_combine in sequence on one stream, with all
+ * intermediates in the workspace. out [T, H] act_dtype. Optional outputs
+ * (NULL to skip): topk_ids [T, k] int32, topk_w [T, k] fp32, counts [E] int32.
+ * shared may be NULL only when cfg->has_shared is 0.
+ */
+int moe_forward(const gbmoe_config* cfg, const void* x, const void* w_router, const float* logit_bias,
+                const float* select_bias, const gbmoe_expert_weights* experts,
+                const gbmoe_expert_weights* shared, void* out, int32_t* topk_ids, float* topk_w,
+                int32_t* counts, void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * moe_forward with HOST activations: copies x_host [T, H] to the device,
+ * runs the layer, copies the result to out_host [T, H] (both act_dtype, on
+ * `stream`, asynchronous: synchronise the stream before reading out_host;
+ * use page-locked host memory for truly asynchronous copies). Weights and the
+ * other arguments are device pointers as in moe_forward.
+ */
+int moe_forward_hostio(const gbmoe_config* cfg, const void* x_host, const void* w_router,
+                       const float* logit_bias, const float* select_bias,
+                       const gbmoe_expert_weights* experts, const gbmoe_expert_weights* shared,
+                       void* out_host, void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * Reads (and clears) the device error word that bounded device-side waits
+ * set in `workspace`, after synchronising `stream`. *status receives GBMOE_OK
+ * or GBMOE_EDEVICE_TIMEOUT. This is the only call that synchronises.
+ */
+int moe_device_status(void* workspace, void* stream, int32_t* status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GBMOE_H */

@@ -1,0 +1,373 @@
+// C ABI of the MoE layer (declared in include/gbmoe.h): argument checks on
+// the host, workspace carving, and the launch sequence of the layer's nodes
+// (MoE Gate -> Fused MoE -> Weight Sum) on the caller's stream.
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+
+#include "common.cuh"
+#include "ffn_sched.h"
+#include "kernels.h"
+
+using namespace gbmoe;
+
+namespace {
+
+constexpr size_t kAlign = 256;
+constexpr int kStreamRowsPerPass = 8;       // matches the streaming kernels' pass height
+constexpr size_t kSmemBudget = 227 * 1024;  // per-CTA shared memory on sm_103a
+constexpr bool kAutoTensorCores = false;    // AUTO picks the tensor-core route once it is validated
+
+size_t align_up(size_t v) { return (v + kAlign - 1) & ~(kAlign - 1); }
+
+size_t act_bytes(int act) { return act == GBMOE_F32 ? 4 : 2; }
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+int check_cfg(const gbmoe_config* c) {
+    if (!c) return GBMOE_EINVAL;
+    if (c->T < 0 || c->H <= 0 || c->I <= 0 || c->E <= 0 || c->top_k <= 0) return GBMOE_EINVAL;
+    if (c->top_k > c->E) return GBMOE_EINVAL;
+    if (c->score != GBMOE_SOFTMAX && c->score != GBMOE_SIGMOID) return GBMOE_EINVAL;
+    if (c->act_dtype != GBMOE_F32 && c->act_dtype != GBMOE_BF16) return GBMOE_EINVAL;
+    if (c->w_dtype < GBMOE_F32 || c->w_dtype > GBMOE_INT4_G128) return GBMOE_EINVAL;
+    if (c->has_shared != 0 && c->has_shared != 1) return GBMOE_EINVAL;
+    if (c->has_shared && c->I_shared <= 0) return GBMOE_EINVAL;
+    if (c->ffn_route < GBMOE_FFN_AUTO || c->ffn_route > GBMOE_FFN_TC) return GBMOE_EINVAL;
+    if (!std::isfinite(c->routed_scale)) return GBMOE_EINVAL;
+    if (c->score == GBMOE_SIGMOID) {
+        if (c->n_group < 1 || c->E % c->n_group != 0) return GBMOE_EINVAL;
+        if (c->n_group > 1 && c->E / c->n_group < 2) return GBMOE_EINVAL;
+        if (c->topk_group < 1 || c->topk_group > c->n_group) return GBMOE_EINVAL;
+        if ((int64_t)c->top_k > (int64_t)c->topk_group * (c->E / c->n_group)) return GBMOE_EINVAL;
+    }
+    // what the kernels cover
+    if (c->H % 256 != 0 || c->I % 128 != 0) return GBMOE_EUNSUPPORTED;
+    if (c->has_shared && c->I_shared % 128 != 0) return GBMOE_EUNSUPPORTED;
+    if (c->E > 512 || c->top_k > 32) return GBMOE_EUNSUPPORTED;
+    if (c->score == GBMOE_SIGMOID && c->n_group > 32) return GBMOE_EUNSUPPORTED;
+    if ((int64_t)c->T * c->top_k > (int64_t(1) << 30)) return GBMOE_EUNSUPPORTED;
+    if (c->act_dtype == GBMOE_BF16 && c->w_dtype == GBMOE_F32) return GBMOE_EUNSUPPORTED;
+    if (c->ffn_route == GBMOE_FFN_TC && c->act_dtype != GBMOE_BF16) return GBMOE_EUNSUPPORTED;
+    return GBMOE_OK;
+}
+
+bool stream_fits(int H, int I, int act) {
+    return (size_t)kStreamRowsPerPass * H * act_bytes(act) <= kSmemBudget &&
+           (size_t)kStreamRowsPerPass * I * act_bytes(act) <= kSmemBudget;
+}
+
+// Kernel route for an FFN problem with n_rows rows over E experts.
+int pick_route(const gbmoe_config* c, int64_t n_rows, int E, int I) {
+    int r = c->ffn_route;
+    if (r != GBMOE_FFN_AUTO) return r;
+    if (n_rows <= 16 * (int64_t)E && stream_fits(c->H, I, c->act_dtype)) return GBMOE_FFN_STREAM;
+    if (c->act_dtype == GBMOE_BF16 && kAutoTensorCores) {
+        FfnProblem probe{};
+        probe.act_dtype = c->act_dtype;
+        probe.w_dtype = c->w_dtype;
+        probe.H = c->H;
+        probe.I = I;
+        probe.E = E;
+        if (ffn_tc_supported(probe)) return GBMOE_FFN_TC;
+    }
+    return GBMOE_FFN_SIMT;
+}
+
+struct Layout {
+    size_t err, logits, ids, w, counts, offsets, sorted, pos, perm, sched, h, xs, y, ysh, xin, xout, total;
+};
+
+Layout layout(const gbmoe_config* c) {
+    const int64_t T = c->T, P = (int64_t)c->T * c->top_k, E = c->E, H = c->H;
+    const size_t ab = act_bytes(c->act_dtype);
+    const int64_t rows_max = P > T ? P : T;
+    const int64_t I_max = c->has_shared && c->I_shared > c->I ? c->I_shared : c->I;
+    Layout L{};
+    size_t o = 0;
+    auto take = [&](size_t bytes) { size_t at = o; o = align_up(o + bytes); return at; };
+    L.err = take(4);
+    L.logits = take((size_t)T * E * 4);
+    L.ids = take((size_t)P * 4);
+    L.w = take((size_t)P * 4);
+    L.counts = take((size_t)E * 4);
+    L.offsets = take((size_t)(E + 1) * 4);
+    L.sorted = take((size_t)P * 4);
+    L.pos = take((size_t)P * 4);
+    L.perm = take(permute_scratch_ints(P, (int)E) * 4);
+    L.sched = take(ffn_sched_ints((int)(E > 1 ? E : 1), rows_max) * 4);
+    L.h = take((size_t)rows_max * I_max * ab);
+    L.xs = take((size_t)rows_max * H * ab);
+    L.y = take((size_t)P * H * ab);
+    L.ysh = take(c->has_shared ? (size_t)T * H * ab : 0);
+    L.xin = take((size_t)T * H * ab);
+    L.xout = take((size_t)T * H * ab);
+    L.total = o;
+    return L;
+}
+
+template <typename T>
+T* at(void* ws, size_t off) {
+    return reinterpret_cast<T*>(static_cast<char*>(ws) + off);
+}
+
+int cuda_status(cudaError_t e) { return e == cudaSuccess ? GBMOE_OK : GBMOE_ECUDA; }
+
+int check_ws(const gbmoe_config* c, void* ws, size_t bytes) {
+    if (!ws || !aligned(ws, kAlign)) return GBMOE_EINVAL;
+    if (bytes < layout(c).total) return GBMOE_EWORKSPACE;
+    return GBMOE_OK;
+}
+
+int check_weights(const gbmoe_config* c, const gbmoe_expert_weights* w) {
+    if (!w || !w->w_gate || !w->w_up || !w->w_down) return GBMOE_EINVAL;
+    if (!aligned(w->w_gate, 16) || !aligned(w->w_up, 16) || !aligned(w->w_down, 16)) return GBMOE_EINVAL;
+    if (c->w_dtype == GBMOE_FP8_E4M3_B128 || c->w_dtype == GBMOE_INT4_G128) {
+        if (!w->s_gate || !w->s_up || !w->s_down) return GBMOE_EINVAL;
+        if (!aligned(w->s_gate, 4) || !aligned(w->s_up, 4) || !aligned(w->s_down, 4)) return GBMOE_EINVAL;
+    }
+    return GBMOE_OK;
+}
+
+RouteParams route_params(const gbmoe_config* c) {
+    RouteParams rp;
+    rp.T = c->T; rp.H = c->H; rp.E = c->E; rp.top_k = c->top_k;
+    rp.score = c->score; rp.renormalize = c->renormalize; rp.n_group = c->n_group;
+    rp.topk_group = c->topk_group; rp.routed_scale = c->routed_scale; rp.act_dtype = c->act_dtype;
+    return rp;
+}
+
+int run_ffn(const gbmoe_config* c, FfnProblem& p, int route, cudaStream_t stream) {
+    cudaError_t err;
+    switch (route) {
+        case GBMOE_FFN_STREAM:
+            if (!stream_fits(p.H, p.I, p.act_dtype)) return GBMOE_EUNSUPPORTED;
+            err = launch_ffn_stream(p, stream);
+            break;
+        case GBMOE_FFN_SIMT: err = launch_ffn_simt(p, stream); break;
+        case GBMOE_FFN_TC:
+            if (!ffn_tc_supported(p)) return GBMOE_EUNSUPPORTED;
+            err = launch_ffn_tc(p, stream);
+            break;
+        default: return GBMOE_EINVAL;
+    }
+    (void)c;
+    return cuda_status(err);
+}
+
+FfnProblem routed_problem(const gbmoe_config* c, const void* x, const int32_t* counts, const int32_t* offsets,
+                          const int32_t* sorted_pair, const gbmoe_expert_weights* w, void* y, void* ws) {
+    const Layout L = layout(c);
+    FfnProblem p{};
+    p.x = x; p.counts = counts; p.offsets = offsets; p.sorted_pair = sorted_pair; p.pair_div = c->top_k;
+    p.E = c->E; p.H = c->H; p.I = c->I; p.n_rows = (int64_t)c->T * c->top_k;
+    p.act_dtype = c->act_dtype; p.w_dtype = c->w_dtype;
+    p.w_gate = w->w_gate; p.w_up = w->w_up; p.w_down = w->w_down;
+    p.s_gate = w->s_gate; p.s_up = w->s_up; p.s_down = w->s_down;
+    p.y = y;
+    p.h = at<char>(ws, L.h); p.x_sorted = at<char>(ws, L.xs); p.sched = at<int32_t>(ws, L.sched);
+    p.err = at<int32_t>(ws, L.err);
+    return p;
+}
+
+FfnProblem shared_problem(const gbmoe_config* c, const void* x, const gbmoe_expert_weights* w, void* y, void* ws) {
+    const Layout L = layout(c);
+    FfnProblem p{};
+    p.x = x; p.counts = nullptr; p.offsets = nullptr; p.sorted_pair = nullptr; p.pair_div = 1;
+    p.E = 1; p.H = c->H; p.I = c->I_shared; p.n_rows = c->T;
+    p.act_dtype = c->act_dtype; p.w_dtype = c->w_dtype;
+    p.w_gate = w->w_gate; p.w_up = w->w_up; p.w_down = w->w_down;
+    p.s_gate = w->s_gate; p.s_up = w->s_up; p.s_down = w->s_down;
+    p.y = y;
+    p.h = at<char>(ws, L.h); p.x_sorted = at<char>(ws, L.xs); p.sched = at<int32_t>(ws, L.sched);
+    p.err = at<int32_t>(ws, L.err);
+    return p;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* gbmoe_status_string(int s) {
+    switch (s) {
+        case GBMOE_OK: return "ok";
+        case GBMOE_EINVAL: return "invalid argument";
+        case GBMOE_EUNSUPPORTED: return "configuration not supported by the kernels";
+        case GBMOE_EWORKSPACE: return "workspace too small";
+        case GBMOE_ECUDA: return "CUDA launch or copy failed";
+        case GBMOE_EDEVICE_TIMEOUT: return "device-side wait timed out";
+        default: return "unknown status";
+    }
+}
+
+int gbmoe_check_config(const gbmoe_config* cfg) { return check_cfg(cfg); }
+
+size_t gbmoe_workspace_size(const gbmoe_config* cfg) {
+    if (check_cfg(cfg) != GBMOE_OK) return 0;
+    return layout(cfg).total;
+}
+
+int moe_route(const gbmoe_config* cfg, const void* x, const void* w_router, const float* logit_bias,
+              const float* select_bias, int32_t* topk_ids, float* topk_w, void* ws, size_t ws_bytes,
+              void* stream) {
+    int s = check_cfg(cfg);
+    if (s) return s;
+    if (cfg->T == 0) return check_ws(cfg, ws, ws_bytes);
+    if (!x || !w_router || !topk_ids || !topk_w) return GBMOE_EINVAL;
+    if (!aligned(x, 16) || !aligned(w_router, 16) || !aligned(topk_ids, 4) || !aligned(topk_w, 4))
+        return GBMOE_EINVAL;
+    if ((logit_bias && !aligned(logit_bias, 4)) || (select_bias && !aligned(select_bias, 4))) return GBMOE_EINVAL;
+    if ((s = check_ws(cfg, ws, ws_bytes))) return s;
+    const Layout L = layout(cfg);
+    return cuda_status(launch_route(route_params(cfg), x, w_router, logit_bias, select_bias, at<float>(ws, L.logits),
+                                    topk_ids, topk_w, static_cast<cudaStream_t>(stream)));
+}
+
+int moe_permute(const gbmoe_config* cfg, const int32_t* topk_ids, int32_t* counts, int32_t* offsets,
+                int32_t* sorted_pair, int32_t* pair_pos, void* ws, size_t ws_bytes, void* stream) {
+    int s = check_cfg(cfg);
+    if (s) return s;
+    if (!topk_ids || !counts || !offsets || !sorted_pair || !pair_pos) return GBMOE_EINVAL;
+    if (!aligned(topk_ids, 4) || !aligned(counts, 4) || !aligned(offsets, 4) || !aligned(sorted_pair, 4) ||
+        !aligned(pair_pos, 4))
+        return GBMOE_EINVAL;
+    if ((s = check_ws(cfg, ws, ws_bytes))) return s;
+    const Layout L = layout(cfg);
+    return cuda_status(launch_permute(topk_ids, (int64_t)cfg->T * cfg->top_k, cfg->E, counts, offsets, sorted_pair,
+                                      pair_pos, at<int32_t>(ws, L.perm), static_cast<cudaStream_t>(stream)));
+}
+
+int moe_grouped_ffn(const gbmoe_config* cfg, const void* x, const int32_t* counts, const int32_t* offsets,
+                    const int32_t* sorted_pair, const gbmoe_expert_weights* experts, void* y_pairs, void* ws,
+                    size_t ws_bytes, void* stream) {
+    int s = check_cfg(cfg);
+    if (s) return s;
+    if (!x || !counts || !offsets || !sorted_pair || !y_pairs) return GBMOE_EINVAL;
+    if (!aligned(x, 16) || !aligned(y_pairs, 16) || !aligned(counts, 4) || !aligned(offsets, 4) ||
+        !aligned(sorted_pair, 4))
+        return GBMOE_EINVAL;
+    if ((s = check_weights(cfg, experts))) return s;
+    if ((s = check_ws(cfg, ws, ws_bytes))) return s;
+    if (cfg->T == 0) return GBMOE_OK;
+    FfnProblem p = routed_problem(cfg, x, counts, offsets, sorted_pair, experts, y_pairs, ws);
+    return run_ffn(cfg, p, pick_route(cfg, p.n_rows, cfg->E, cfg->I), static_cast<cudaStream_t>(stream));
+}
+
+int moe_shared_ffn(const gbmoe_config* cfg, const void* x, const gbmoe_expert_weights* shared, void* y_shared,
+                   void* ws, size_t ws_bytes, void* stream) {
+    int s = check_cfg(cfg);
+    if (s) return s;
+    if (!cfg->has_shared || !x || !y_shared || !aligned(x, 16) || !aligned(y_shared, 16)) return GBMOE_EINVAL;
+    if ((s = check_weights(cfg, shared))) return s;
+    if ((s = check_ws(cfg, ws, ws_bytes))) return s;
+    if (cfg->T == 0) return GBMOE_OK;
+    FfnProblem p = shared_problem(cfg, x, shared, y_shared, ws);
+    return run_ffn(cfg, p, pick_route(cfg, cfg->T, 1, cfg->I_shared), static_cast<cudaStream_t>(stream));
+}
+
+int moe_combine(const gbmoe_config* cfg, const void* y_pairs, const float* topk_w, const int32_t* pair_pos,
+                const void* y_shared, void* out, void* stream) {
+    int s = check_cfg(cfg);
+    if (s) return s;
+    if (cfg->T == 0) return GBMOE_OK;
+    if (!y_pairs || !topk_w || !pair_pos || !out) return GBMOE_EINVAL;
+    if (!aligned(y_pairs, 16) || !aligned(out, 16) || !aligned(topk_w, 4) || !aligned(pair_pos, 4) ||
+        (y_shared && !aligned(y_shared, 16)))
+        return GBMOE_EINVAL;
+    return cuda_status(launch_combine(y_pairs, topk_w, pair_pos, y_shared, out, cfg->T, cfg->top_k, cfg->H,
+                                      cfg->act_dtype, static_cast<cudaStream_t>(stream)));
+}
+
+int moe_forward(const gbmoe_config* cfg, const void* x, const void* w_router, const float* logit_bias,
+                const float* select_bias, const gbmoe_expert_weights* experts, const gbmoe_expert_weights* shared,
+                void* out, int32_t* topk_ids, float* topk_w, int32_t* counts_out, void* ws, size_t ws_bytes,
+                void* stream) {
+    int s = check_cfg(cfg);
+    if (s) return s;
+    if (cfg->T == 0) return check_ws(cfg, ws, ws_bytes);  // nothing to read or write
+    if (!x || !w_router || !out || !aligned(x, 16) || !aligned(w_router, 16) || !aligned(out, 16))
+        return GBMOE_EINVAL;
+    if ((logit_bias && !aligned(logit_bias, 4)) || (select_bias && !aligned(select_bias, 4))) return GBMOE_EINVAL;
+    if ((topk_ids && !aligned(topk_ids, 4)) || (topk_w && !aligned(topk_w, 4)) ||
+        (counts_out && !aligned(counts_out, 4)))
+        return GBMOE_EINVAL;
+    if ((s = check_weights(cfg, experts))) return s;
+    if (cfg->has_shared && (s = check_weights(cfg, shared))) return s;
+    if ((s = check_ws(cfg, ws, ws_bytes))) return s;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const Layout L = layout(cfg);
+    const int64_t P = (int64_t)cfg->T * cfg->top_k;
+    // every route must be launchable before anything is enqueued
+    const int r_routed = pick_route(cfg, P, cfg->E, cfg->I);
+    const int r_shared = cfg->has_shared ? pick_route(cfg, cfg->T, 1, cfg->I_shared) : GBMOE_FFN_SIMT;
+    for (int r : {r_routed, r_shared}) {
+        if (r == GBMOE_FFN_STREAM && !stream_fits(cfg->H, r == r_routed ? cfg->I : cfg->I_shared, cfg->act_dtype))
+            return GBMOE_EUNSUPPORTED;
+    }
+    if (cudaMemsetAsync(at<int32_t>(ws, L.err), 0, 4, st) != cudaSuccess) return GBMOE_ECUDA;
+    if (cfg->T == 0) return GBMOE_OK;
+    int32_t* ids = at<int32_t>(ws, L.ids);
+    float* w = at<float>(ws, L.w);
+    int32_t* counts = at<int32_t>(ws, L.counts);
+    int32_t* offsets = at<int32_t>(ws, L.offsets);
+    int32_t* sorted = at<int32_t>(ws, L.sorted);
+    int32_t* pos = at<int32_t>(ws, L.pos);
+    if ((s = cuda_status(launch_route(route_params(cfg), x, w_router, logit_bias, select_bias,
+                                      at<float>(ws, L.logits), ids, w, st))))
+        return s;
+    if ((s = cuda_status(launch_permute(ids, P, cfg->E, counts, offsets, sorted, pos, at<int32_t>(ws, L.perm), st))))
+        return s;
+    void* y = at<char>(ws, L.y);
+    FfnProblem pr = routed_problem(cfg, x, counts, offsets, sorted, experts, y, ws);
+    if ((s = run_ffn(cfg, pr, r_routed, st))) return s;
+    void* ysh = nullptr;
+    if (cfg->has_shared) {
+        ysh = at<char>(ws, L.ysh);
+        FfnProblem ps = shared_problem(cfg, x, shared, ysh, ws);
+        if ((s = run_ffn(cfg, ps, r_shared, st))) return s;
+    }
+    if ((s = cuda_status(launch_combine(y, w, pos, ysh, out, cfg->T, cfg->top_k, cfg->H, cfg->act_dtype, st))))
+        return s;
+    if (topk_ids && cudaMemcpyAsync(topk_ids, ids, P * 4, cudaMemcpyDeviceToDevice, st) != cudaSuccess)
+        return GBMOE_ECUDA;
+    if (topk_w && cudaMemcpyAsync(topk_w, w, P * 4, cudaMemcpyDeviceToDevice, st) != cudaSuccess) return GBMOE_ECUDA;
+    if (counts_out && cudaMemcpyAsync(counts_out, counts, (size_t)cfg->E * 4, cudaMemcpyDeviceToDevice, st) !=
+                          cudaSuccess)
+        return GBMOE_ECUDA;
+    return GBMOE_OK;
+}
+
+int moe_forward_hostio(const gbmoe_config* cfg, const void* x_host, const void* w_router, const float* logit_bias,
+                       const float* select_bias, const gbmoe_expert_weights* experts,
+                       const gbmoe_expert_weights* shared, void* out_host, void* ws, size_t ws_bytes, void* stream) {
+    int s = check_cfg(cfg);
+    if (s) return s;
+    if ((s = check_ws(cfg, ws, ws_bytes))) return s;
+    if (cfg->T == 0) return GBMOE_OK;
+    if (!x_host || !out_host) return GBMOE_EINVAL;
+    const Layout L = layout(cfg);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const size_t bytes = (size_t)cfg->T * cfg->H * act_bytes(cfg->act_dtype);
+    void* xin = at<char>(ws, L.xin);
+    void* xout = at<char>(ws, L.xout);
+    if (bytes && cudaMemcpyAsync(xin, x_host, bytes, cudaMemcpyHostToDevice, st) != cudaSuccess) return GBMOE_ECUDA;
+    s = moe_forward(cfg, xin, w_router, logit_bias, select_bias, experts, shared, xout, nullptr, nullptr, nullptr, ws,
+                    ws_bytes, stream);
+    if (s) return s;
+    if (bytes && cudaMemcpyAsync(out_host, xout, bytes, cudaMemcpyDeviceToHost, st) != cudaSuccess)
+        return GBMOE_ECUDA;
+    return GBMOE_OK;
+}
+
+int moe_device_status(void* ws, void* stream, int32_t* status) {
+    if (!ws || !status || !aligned(ws, kAlign)) return GBMOE_EINVAL;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    int32_t word = 0;
+    if (cudaStreamSynchronize(st) != cudaSuccess) return GBMOE_ECUDA;
+    if (cudaMemcpy(&word, ws, 4, cudaMemcpyDeviceToHost) != cudaSuccess) return GBMOE_ECUDA;
+    if (cudaMemset(ws, 0, 4) != cudaSuccess) return GBMOE_ECUDA;
+    *status = word ? GBMOE_EDEVICE_TIMEOUT : GBMOE_OK;
+    return GBMOE_OK;
+}
+
+}  // extern "C"

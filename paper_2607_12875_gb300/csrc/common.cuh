@@ -1,0 +1,114 @@
+// Shared device helpers for the MoE layer kernels (sm_103a).
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/gbmoe.h"
+
+namespace gbmoe {
+
+constexpr int kWarp = 32;
+
+__host__ __device__ __forceinline__ int64_t min64(int64_t a, int64_t b) { return a < b ? a : b; }
+
+// ------------------------------------------------------------ bf16 helpers
+
+__device__ __forceinline__ float bf16lo(uint32_t v) { return __uint_as_float(v << 16); }
+__device__ __forceinline__ float bf16hi(uint32_t v) { return __uint_as_float(v & 0xffff0000u); }
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+    __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);  // .x = lo, .y = hi, RNE
+    return *reinterpret_cast<uint32_t*>(&h);
+}
+
+// Eight consecutive activation elements starting at p (16-byte aligned for
+// bf16, 32-byte aligned for fp32) widened to fp32.
+template <typename TA>
+struct Vec8;
+
+template <>
+struct Vec8<__nv_bfloat16> {
+    __device__ __forceinline__ static void load(const __nv_bfloat16* p, float (&v)[8]) {
+        uint4 u = *reinterpret_cast<const uint4*>(p);
+        v[0] = bf16lo(u.x); v[1] = bf16hi(u.x); v[2] = bf16lo(u.y); v[3] = bf16hi(u.y);
+        v[4] = bf16lo(u.z); v[5] = bf16hi(u.z); v[6] = bf16lo(u.w); v[7] = bf16hi(u.w);
+    }
+    __device__ __forceinline__ static void store(__nv_bfloat16* p, const float (&v)[8]) {
+        uint4 u;
+        u.x = pack_bf16x2(v[0], v[1]); u.y = pack_bf16x2(v[2], v[3]);
+        u.z = pack_bf16x2(v[4], v[5]); u.w = pack_bf16x2(v[6], v[7]);
+        *reinterpret_cast<uint4*>(p) = u;
+    }
+};
+
+template <>
+struct Vec8<float> {
+    __device__ __forceinline__ static void load(const float* p, float (&v)[8]) {
+        float4 a = *reinterpret_cast<const float4*>(p);
+        float4 b = *reinterpret_cast<const float4*>(p + 4);
+        v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+    }
+    __device__ __forceinline__ static void store(float* p, const float (&v)[8]) {
+        *reinterpret_cast<float4*>(p) = make_float4(v[0], v[1], v[2], v[3]);
+        *reinterpret_cast<float4*>(p + 4) = make_float4(v[4], v[5], v[6], v[7]);
+    }
+};
+
+template <typename T>
+__device__ __forceinline__ float to_f32(T v);
+template <>
+__device__ __forceinline__ float to_f32<float>(float v) { return v; }
+template <>
+__device__ __forceinline__ float to_f32<__nv_bfloat16>(__nv_bfloat16 v) { return __bfloat162float(v); }
+
+template <typename T>
+__device__ __forceinline__ T from_f32(float v);
+template <>
+__device__ __forceinline__ float from_f32<float>(float v) { return v; }
+template <>
+__device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float v) { return __float2bfloat16_rn(v); }
+
+// 16-byte load of data read once (expert weights): not kept in L1.
+__device__ __forceinline__ uint4 ld_stream16(const void* p) {
+    uint4 r;
+    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+                 : "l"(p));
+    return r;
+}
+
+// ------------------------------------------------------- weight decoding
+
+// e4m3 byte -> fp32 value (sign, 4-bit exponent with bias 7, 3-bit mantissa,
+// subnormals at exponent 0; the NaN code is never produced by a quantiser).
+__device__ __forceinline__ float e4m3_to_f32(uint32_t b) {
+    uint32_t sign = (b & 0x80u) << 24;
+    uint32_t em = b & 0x7fu;
+    float mag;
+    if (em >= 8u) {
+        // normal: rebias exponent 7 -> 127, mantissa 3 -> 23 bits
+        mag = __uint_as_float(((em >> 3) + 120u) << 23 | (em & 7u) << 20);
+    } else {
+        mag = (float)em * 0.001953125f;  // m * 2^-9
+    }
+    return __uint_as_float(__float_as_uint(mag) | sign);
+}
+
+// signed 4-bit value of nibble n (two's complement)
+__device__ __forceinline__ float int4_to_f32(uint32_t n) { return (float)((int32_t)(n << 28) >> 28); }
+
+// ------------------------------------------------------------- silu
+
+__device__ __forceinline__ float silu_mul(float g, float u) { return g / (1.0f + expf(-g)) * u; }
+
+// ------------------------------------------------------------ errors
+
+constexpr int32_t kErrTimeout = 1;
+
+__device__ __forceinline__ void set_error(int32_t* err, int32_t code) {
+    if (err) atomicOr(err, code);
+}
+
+}  // namespace gbmoe

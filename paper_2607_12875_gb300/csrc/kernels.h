@@ -1,0 +1,57 @@
+// Internal launch interface between the C ABI (api.cu) and the kernels.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace gbmoe {
+
+struct RouteParams {
+    int T, H, E, top_k;
+    int score, renormalize, n_group, topk_group;
+    float routed_scale;
+    int act_dtype;
+};
+
+// logits [T, E] fp32 scratch; topk_ids, topk_w [T, k]
+cudaError_t launch_route(const RouteParams& rp, const void* x, const void* w_router, const float* logit_bias,
+                         const float* select_bias, float* logits, int32_t* topk_ids, float* topk_w,
+                         cudaStream_t stream);
+
+// Number of 1024-pair blocks the permutation uses, and its scratch ints.
+int permute_blocks(int64_t P);
+size_t permute_scratch_ints(int64_t P, int E);
+cudaError_t launch_permute(const int32_t* topk_ids, int64_t P, int E, int32_t* counts, int32_t* offsets,
+                           int32_t* sorted_pair, int32_t* pair_pos, int32_t* scratch, cudaStream_t stream);
+
+// One grouped FFN problem: rows r of expert e are offsets[e] .. offsets[e+1]-1,
+// the token of row r is sorted_pair[r] / pair_div (r itself when sorted_pair
+// is null). counts null means one expert with n_rows rows.
+struct FfnProblem {
+    const void* x;              // [T, H] act
+    const int32_t* counts;      // [E] or null
+    const int32_t* offsets;     // [E+1] or null (then 0, n_rows)
+    const int32_t* sorted_pair; // [rows] or null
+    int pair_div;
+    int E, H, I;
+    int64_t n_rows;             // upper bound on rows (P, or T for the shared expert)
+    int act_dtype, w_dtype;
+    const void *w_gate, *w_up, *w_down, *s_gate, *s_up, *s_down;
+    void* y;                    // [n_rows, H] act
+    // scratch carved by the caller
+    void* h;                    // [n_rows, I] act
+    void* x_sorted;             // [n_rows, H] act (tensor-core route only)
+    int32_t* sched;             // schedule ints, ffn_sched_ints(E, n_rows)
+    int32_t* err;               // device error word
+};
+
+size_t ffn_sched_ints(int E, int64_t n_rows);
+cudaError_t launch_ffn_stream(const FfnProblem& p, cudaStream_t stream);
+cudaError_t launch_ffn_simt(const FfnProblem& p, cudaStream_t stream);
+cudaError_t launch_ffn_tc(const FfnProblem& p, cudaStream_t stream);
+bool ffn_tc_supported(const FfnProblem& p);
+
+cudaError_t launch_combine(const void* y_pairs, const float* topk_w, const int32_t* pair_pos, const void* y_shared,
+                           void* out, int T, int k, int H, int act_dtype, cudaStream_t stream);
+
+}  // namespace gbmoe

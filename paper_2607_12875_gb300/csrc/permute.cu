@@ -1,0 +1,121 @@
+// Fused MoE, grouping step: stable counting sort of the (token, slot) pairs
+// by expert. Three small kernels: per-block histograms, one scan that turns
+// them into counts, offsets and per-block bases, and a scatter that ranks
+// pairs inside a block in pair order (warp match + warp-ordered running
+// counters), so the result is the stable order whatever the scheduling.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace gbmoe {
+
+constexpr int kPermBlock = 1024;  // pairs per block (one per thread)
+
+int permute_blocks(int64_t P) { return (int)((P + kPermBlock - 1) / kPermBlock); }
+
+// block histograms [nblk][E] + per-block bases [nblk][E]
+size_t permute_scratch_ints(int64_t P, int E) { return 2 * (size_t)permute_blocks(P) * E; }
+
+__global__ void __launch_bounds__(kPermBlock)
+perm_hist_kernel(const int32_t* __restrict__ ids, int64_t P, int E, int32_t* __restrict__ block_hist) {
+    extern __shared__ int32_t s_hist[];
+    for (int e = threadIdx.x; e < E; e += blockDim.x) s_hist[e] = 0;
+    __syncthreads();
+    int64_t p = (int64_t)blockIdx.x * kPermBlock + threadIdx.x;
+    if (p < P) {
+        const int e = ids[p];
+        if (e >= 0 && e < E) atomicAdd(&s_hist[e], 1);  // out-of-range ids are dropped
+    }
+    __syncthreads();
+    for (int e = threadIdx.x; e < E; e += blockDim.x) block_hist[(size_t)blockIdx.x * E + e] = s_hist[e];
+}
+
+// One block, thread e owns expert e: walks the block histograms in order.
+__global__ void __launch_bounds__(512)
+perm_scan_kernel(const int32_t* __restrict__ block_hist, int nblk, int E, int32_t* __restrict__ counts,
+                 int32_t* __restrict__ offsets, int32_t* __restrict__ block_base) {
+    __shared__ int32_t s_warp[16];
+    const int e = threadIdx.x;
+    int run = 0;
+    if (e < E)
+        for (int b = 0; b < nblk; ++b) {
+            block_base[(size_t)b * E + e] = run;
+            run += block_hist[(size_t)b * E + e];
+        }
+    // exclusive scan of the counts over experts
+    const int lane = e & 31, warp = e >> 5;
+    int v = (e < E) ? run : 0, incl = v;
+#pragma unroll
+    for (int d = 1; d < 32; d <<= 1) {
+        int o = __shfl_up_sync(0xffffffffu, incl, d);
+        if (lane >= d) incl += o;
+    }
+    if (lane == 31) s_warp[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+        int w = (lane < (int)(blockDim.x >> 5)) ? s_warp[lane] : 0, wi = w;
+#pragma unroll
+        for (int d = 1; d < 32; d <<= 1) {
+            int o = __shfl_up_sync(0xffffffffu, wi, d);
+            if (lane >= d) wi += o;
+        }
+        if (lane < 16) s_warp[lane] = wi - w;  // exclusive warp prefix
+    }
+    __syncthreads();
+    int excl = s_warp[warp] + incl - v;
+    if (e < E) {
+        counts[e] = run;
+        offsets[e] = excl;
+        if (e == E - 1) offsets[E] = excl + run;
+        for (int b = 0; b < nblk; ++b) block_base[(size_t)b * E + e] += excl;
+    }
+}
+
+__global__ void __launch_bounds__(kPermBlock)
+perm_scatter_kernel(const int32_t* __restrict__ ids, int64_t P, int E, const int32_t* __restrict__ block_base,
+                    int32_t* __restrict__ sorted_pair, int32_t* __restrict__ pair_pos) {
+    extern __shared__ int32_t s_run[];
+    for (int e = threadIdx.x; e < E; e += blockDim.x) s_run[e] = block_base[(size_t)blockIdx.x * E + e];
+    __syncthreads();
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int64_t p = (int64_t)blockIdx.x * kPermBlock + threadIdx.x;
+    const int id = p < P ? ids[p] : -1;
+    const bool valid = id >= 0 && id < E;
+    const int e = valid ? id : -1 - lane;  // invalid lanes never match a real expert
+    const uint32_t peers = __match_any_sync(0xffffffffu, e);
+    const int rank = __popc(peers & ((1u << lane) - 1u));
+    const bool leader = rank == 0;
+    int pos = 0;
+    // warps take their places in pair order
+    for (int w = 0; w < kPermBlock / 32; ++w) {
+        if (warp == w && valid) {
+            pos = s_run[e] + rank;
+            __syncwarp(peers);
+            if (leader) s_run[e] += __popc(peers);
+        }
+        __syncthreads();
+    }
+    if (valid) {
+        sorted_pair[pos] = (int32_t)p;
+        pair_pos[p] = pos;
+    }
+}
+
+cudaError_t launch_permute(const int32_t* topk_ids, int64_t P, int E, int32_t* counts, int32_t* offsets,
+                           int32_t* sorted_pair, int32_t* pair_pos, int32_t* scratch, cudaStream_t stream) {
+    const int nblk = permute_blocks(P);
+    int32_t* block_hist = scratch;
+    int32_t* block_base = scratch + (size_t)nblk * E;
+    if (nblk > 0) {
+        perm_hist_kernel<<<nblk, kPermBlock, E * sizeof(int32_t), stream>>>(topk_ids, P, E, block_hist);
+        cudaError_t err = cudaGetLastError();
+        if (err != cudaSuccess) return err;
+    }
+    perm_scan_kernel<<<1, 512, 0, stream>>>(block_hist, nblk, E, counts, offsets, block_base);
+    cudaError_t err = cudaGetLastError();
+    if (err != cudaSuccess || nblk == 0) return err;
+    perm_scatter_kernel<<<nblk, kPermBlock, E * sizeof(int32_t), stream>>>(topk_ids, P, E, block_base,
+                                                                           sorted_pair, pair_pos);
+    return cudaGetLastError();
+}
+
+}  // namespace gbmoe

@@ -1,0 +1,261 @@
+// MoE Gate: router logits, expert choice and routing weights.
+//
+// Two kernels. gate_logits computes l[t,e] = x[t,:].Wg[e,:] (+ bias[e]) in
+// fp32 in the fixed order the layer's definition uses (32 partial sums over
+// interleaved 8-element chunks, one fused multiply-add per element, then a
+// butterfly of pairwise sums), so the expert choice is bit-identical to the
+// oracle's. A warp owns TB tokens x 8 experts; lane l holds the partial sums
+// of chunks l, l+32, ... for all of them, which is exactly the fixed order.
+// select_experts then runs one warp per token over the logits.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace gbmoe {
+
+constexpr int kGateWarps = 8;
+constexpr int kGateExpertsPerWarp = 8;
+
+template <typename TA, int TB>
+__global__ void __launch_bounds__(kGateWarps * 32)
+gate_logits_kernel(const TA* __restrict__ x, const TA* __restrict__ wg, const float* __restrict__ bias,
+                   float* __restrict__ logits, int T, int H, int E) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int t0 = blockIdx.x * TB;
+    const int e0 = (blockIdx.y * kGateWarps + warp) * kGateExpertsPerWarp;
+    if (e0 >= E) return;
+    float acc[TB][kGateExpertsPerWarp];
+#pragma unroll
+    for (int a = 0; a < TB; ++a)
+#pragma unroll
+        for (int b = 0; b < kGateExpertsPerWarp; ++b) acc[a][b] = 0.0f;
+
+    const int nchunk = H / 8;  // H % 256 == 0: every lane gets H/256 chunks
+    for (int c = lane; c < nchunk; c += 32) {
+        float xv[TB][8];
+#pragma unroll
+        for (int a = 0; a < TB; ++a) {
+            int t = t0 + a;
+            if (t < T) {
+                Vec8<TA>::load(x + (size_t)t * H + 8 * c, xv[a]);
+            } else {
+#pragma unroll
+                for (int i = 0; i < 8; ++i) xv[a][i] = 0.0f;
+            }
+        }
+#pragma unroll
+        for (int b = 0; b < kGateExpertsPerWarp; ++b) {
+            int e = e0 + b;
+            float wv[8];
+            if (e < E) {
+                Vec8<TA>::load(wg + (size_t)e * H + 8 * c, wv);
+            } else {
+#pragma unroll
+                for (int i = 0; i < 8; ++i) wv[i] = 0.0f;
+            }
+#pragma unroll
+            for (int a = 0; a < TB; ++a)
+#pragma unroll
+                for (int i = 0; i < 8; ++i) acc[a][b] = __fmaf_rn(xv[a][i], wv[i], acc[a][b]);
+        }
+    }
+    // butterfly: s[p] <- s[p] + s[p ^ d], d = 16 .. 1 (one commutative add: all lanes end equal)
+#pragma unroll
+    for (int a = 0; a < TB; ++a)
+#pragma unroll
+        for (int b = 0; b < kGateExpertsPerWarp; ++b) {
+            float v = acc[a][b];
+#pragma unroll
+            for (int d = 16; d >= 1; d >>= 1) v = __fadd_rn(v, __shfl_xor_sync(0xffffffffu, v, d));
+            acc[a][b] = v;
+        }
+#pragma unroll
+    for (int a = 0; a < TB; ++a)
+#pragma unroll
+        for (int b = 0; b < kGateExpertsPerWarp; ++b) {
+            int t = t0 + a, e = e0 + b;
+            if (lane == ((a * kGateExpertsPerWarp + b) & 31) && t < T && e < E) {
+                float l = acc[a][b];
+                if (bias) l = __fadd_rn(l, bias[e]);
+                logits[(size_t)t * E + e] = l;
+            }
+        }
+}
+
+// ------------------------------------------------------- expert choice
+
+// Fixed fp32 exponential for the sigmoid score (the expert choice depends on
+// its exact bits, so it is not left to a library): clamp to [-86, 88];
+// n = rint(x*log2 e); r = (x - n*ln2_hi) - n*ln2_lo with ln2_hi the leading
+// 16 bits of ln 2 (Cody-Waite reduction, exact n*ln2_hi); exp(r) from its
+// degree-8 Taylor polynomial by Horner's rule, a separate rounded multiply
+// and add per step; times 2^n assembled from exponent bits.
+__device__ __forceinline__ float pinned_exp(float x) {
+    const float kLog2e = __uint_as_float(0x3fb8aa3bu);  // fp32(1/ln 2)
+    const float kLn2Hi = __uint_as_float(0x3f317200u);  // 0.693145751953125
+    const float kLn2Lo = __uint_as_float(0x35bfbe8eu);  // fp32(ln 2 - kLn2Hi)
+    const uint32_t kInvFact[9] = {0x3f800000u, 0x3f800000u, 0x3f000000u, 0x3e2aaaabu, 0x3d2aaaabu,
+                                  0x3c088889u, 0x3ab60b61u, 0x39500d01u, 0x37d00d01u};  // fp32(1/i!)
+    x = fminf(fmaxf(x, -86.0f), 88.0f);
+    float n = rintf(__fmul_rn(x, kLog2e));
+    float r = __fsub_rn(x, __fmul_rn(n, kLn2Hi));
+    r = __fsub_rn(r, __fmul_rn(n, kLn2Lo));
+    float p = __uint_as_float(kInvFact[8]);
+#pragma unroll
+    for (int i = 7; i >= 0; --i) p = __fadd_rn(__fmul_rn(p, r), __uint_as_float(kInvFact[i]));
+    return __fmul_rn(p, __uint_as_float((uint32_t)((int)n + 127) << 23));
+}
+
+__device__ __forceinline__ float pinned_sigmoid(float l) {
+    return __fdiv_rn(1.0f, __fadd_rn(1.0f, pinned_exp(-l)));
+}
+
+// (key, index) with "larger key, then smaller index" as the better candidate
+__device__ __forceinline__ bool better(float ka, int ia, float kb, int ib) {
+    return ka > kb || (ka == kb && ia < ib);
+}
+
+__device__ __forceinline__ void warp_best(float& k, int& i) {
+#pragma unroll
+    for (int d = 16; d >= 1; d >>= 1) {
+        float ko = __shfl_xor_sync(0xffffffffu, k, d);
+        int io = __shfl_xor_sync(0xffffffffu, i, d);
+        if (better(ko, io, k, i)) { k = ko; i = io; }
+    }
+}
+
+constexpr int kSelWarps = 4;
+constexpr int kMaxE = 512;
+
+// One warp per token. Expert e lives in lane e % 32, slot e / 32.
+__global__ void __launch_bounds__(kSelWarps * 32)
+select_experts_kernel(const float* __restrict__ logits, const float* __restrict__ select_bias,
+                      int32_t* __restrict__ topk_ids, float* __restrict__ topk_w, RouteParams rp) {
+    __shared__ float s_key[kSelWarps][kMaxE];
+    __shared__ float s_sig[kSelWarps][kMaxE];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int t = blockIdx.x * kSelWarps + warp;
+    if (t >= rp.T) return;
+    const int E = rp.E, k = rp.top_k;
+    const float* l = logits + (size_t)t * E;
+    float* key = s_key[warp];
+    float* sig = s_sig[warp];
+    const bool sigmoid = rp.score == GBMOE_SIGMOID;
+    for (int e = lane; e < E; e += 32) {
+        float v = l[e];
+        if (sigmoid) {
+            float s = pinned_sigmoid(v);
+            sig[e] = s;
+            v = select_bias ? __fadd_rn(s, select_bias[e]) : s;
+        }
+        key[e] = v;
+    }
+    __syncwarp();
+
+    // groups kept (bit g set); all experts allowed without group limiting
+    uint32_t kept = 0xffffffffu;
+    const int G = sigmoid ? rp.n_group : 1;
+    if (G > 1) {
+        const int gs = E / G;
+        float gscore = -INFINITY;
+        if (lane < G) {
+            float a = -INFINITY, b = -INFINITY;  // two largest q of group `lane`
+            for (int e = lane * gs; e < (lane + 1) * gs; ++e) {
+                float v = key[e];
+                if (v > a) { b = a; a = v; } else if (v > b) { b = v; }
+            }
+            gscore = __fadd_rn(a, b);
+        }
+        kept = 0u;
+        bool taken = false;
+        for (int r = 0; r < rp.topk_group; ++r) {
+            float kk = (lane < G && !taken) ? gscore : -INFINITY;
+            int ii = (lane < G && !taken) ? lane : 0x7fffffff;
+            warp_best(kk, ii);
+            kept |= 1u << ii;
+            if (lane == ii) taken = true;
+        }
+    }
+    const int gs = E / G;
+
+    // top-k over allowed experts, descending key, ties to the lower index
+    uint32_t used = 0u;  // bit s: expert lane + 32 s already chosen
+    int sel_id = 0;
+    float top_key = 0.0f;
+    for (int j = 0; j < k; ++j) {
+        float kk = -INFINITY;
+        int ii = 0x7fffffff;
+        for (int s = 0, e = lane; e < E; ++s, e += 32) {
+            if ((used >> s) & 1u) continue;
+            if (!((kept >> (e / gs)) & 1u)) continue;
+            float v = key[e];
+            if (ii == 0x7fffffff || better(v, e, kk, ii)) { kk = v; ii = e; }
+        }
+        warp_best(kk, ii);
+        if ((ii & 31) == lane) used |= 1u << (ii >> 5);
+        if (j == 0) top_key = kk;
+        if (lane == j) sel_id = ii;
+    }
+
+    // routing weights (lane j < k holds slot j)
+    float w = 0.0f;
+    if (!sigmoid) {
+        float lj = (lane < k) ? l[sel_id] : 0.0f;
+        float m = top_key, z = 0.0f;
+        if (!rp.renormalize) {
+            float mm = -INFINITY;
+            for (int e = lane; e < E; e += 32) mm = fmaxf(mm, l[e]);
+#pragma unroll
+            for (int d = 16; d >= 1; d >>= 1) mm = fmaxf(mm, __shfl_xor_sync(0xffffffffu, mm, d));
+            m = mm;
+            for (int e = lane; e < E; e += 32) z += expf(l[e] - m);
+        } else {
+            z = (lane < k) ? expf(lj - m) : 0.0f;
+        }
+#pragma unroll
+        for (int d = 16; d >= 1; d >>= 1) z += __shfl_xor_sync(0xffffffffu, z, d);
+        w = (lane < k) ? expf(lj - m) / z * rp.routed_scale : 0.0f;
+    } else {
+        float sj = (lane < k) ? sig[sel_id] : 0.0f;
+        float z = sj;
+#pragma unroll
+        for (int d = 16; d >= 1; d >>= 1) z += __shfl_xor_sync(0xffffffffu, z, d);
+        w = (rp.renormalize ? sj / z : sj) * rp.routed_scale;
+    }
+    if (lane < k) {
+        topk_ids[(size_t)t * k + lane] = sel_id;
+        topk_w[(size_t)t * k + lane] = w;
+    }
+}
+
+cudaError_t launch_route(const RouteParams& rp, const void* x, const void* wg, const float* logit_bias,
+                         const float* select_bias, float* logits, int32_t* topk_ids, float* topk_w,
+                         cudaStream_t stream) {
+    if (rp.T == 0) return cudaSuccess;
+    const int ey = (rp.E + kGateWarps * kGateExpertsPerWarp - 1) / (kGateWarps * kGateExpertsPerWarp);
+    dim3 block(kGateWarps * 32);
+    if (rp.act_dtype == GBMOE_BF16) {
+        auto xp = static_cast<const __nv_bfloat16*>(x);
+        auto wp = static_cast<const __nv_bfloat16*>(wg);
+        if (rp.T >= 1024) {
+            dim3 grid((rp.T + 7) / 8, ey);
+            gate_logits_kernel<__nv_bfloat16, 8><<<grid, block, 0, stream>>>(xp, wp, logit_bias, logits, rp.T,
+                                                                              rp.H, rp.E);
+        } else {
+            dim3 grid((rp.T + 1) / 2, ey);
+            gate_logits_kernel<__nv_bfloat16, 2><<<grid, block, 0, stream>>>(xp, wp, logit_bias, logits, rp.T,
+                                                                              rp.H, rp.E);
+        }
+    } else {
+        auto xp = static_cast<const float*>(x);
+        auto wp = static_cast<const float*>(wg);
+        dim3 grid((rp.T + 1) / 2, ey);
+        gate_logits_kernel<float, 2><<<grid, block, 0, stream>>>(xp, wp, logit_bias, logits, rp.T, rp.H, rp.E);
+    }
+    cudaError_t err = cudaGetLastError();
+    if (err != cudaSuccess) return err;
+    select_experts_kernel<<<(rp.T + kSelWarps - 1) / kSelWarps, kSelWarps * 32, 0, stream>>>(
+        logits, select_bias, topk_ids, topk_w, rp);
+    return cudaGetLastError();
+}
+
+}  // namespace gbmoe

@@ -1,0 +1,128 @@
+"""CPU checks of the C-ABI library: it loads, exports every function the
+header declares, and rejects bad arguments on the host (no GPU involved:
+every case below returns before any CUDA call)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2607_12875_gb300 as gb
+import synth
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "gbmoe.h")
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return re.findall(r"^[A-Za-z_][\w \t\*]*?\b((?:gbmoe|moe)_\w+)\s*\(", text, flags=re.M)
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if not os.path.exists(gb.LIB_PATH):
+        from paper_2607_12875_gb300 import build
+        build.build()
+    return gb.lib()
+
+
+def test_header_declares_the_layer_entry_points():
+    names = declared_functions()
+    for n in ("moe_route", "moe_permute", "moe_grouped_ffn", "moe_combine", "moe_forward"):
+        assert n in names
+    assert set(names) == set(gb.EXPORTS)
+
+
+def test_library_exports_every_declared_function(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+
+
+def cfg_of(wid, **kw):
+    w = synth.WORKLOADS[wid]
+    c = gb.make_config(w.T, w.H, w.I, w.E, w.top_k, score=w.score, renormalize=w.renormalize, n_group=w.n_group,
+                       topk_group=w.topk_group, routed_scale=w.routed_scale, act=w.act, w=w.wq,
+                       has_shared=w.has_shared, I_shared=w.I_shared)
+    for k, v in kw.items():
+        setattr(c, k, v)
+    return c
+
+
+@pytest.mark.parametrize("wid", [1, 2, 3, 4, 5])
+def test_workload_configs_are_valid(lib, wid):
+    c = cfg_of(wid)
+    assert gb.check_config(c) == gb.OK
+    assert gb.workspace_size(c) > 0
+
+
+@pytest.mark.parametrize("change,status", [
+    (dict(H=300), gb.EUNSUPPORTED),
+    (dict(H=0), gb.EINVAL),
+    (dict(I=100), gb.EUNSUPPORTED),
+    (dict(top_k=9), gb.EINVAL),
+    (dict(E=1024, top_k=2), gb.EUNSUPPORTED),
+    (dict(T=-1), gb.EINVAL),
+    (dict(score=7), gb.EINVAL),
+    (dict(act_dtype=2), gb.EINVAL),
+    (dict(ffn_route=9), gb.EINVAL),
+    (dict(ffn_route=gb.FFN_TC), gb.EUNSUPPORTED),  # fp32 activations have no tensor-core route
+])
+def test_invalid_configs_are_rejected(lib, change, status):
+    c = cfg_of(1, **change)
+    assert gb.check_config(c) == status
+    assert gb.workspace_size(c) == 0
+
+
+def test_sigmoid_group_rules(lib):
+    c = cfg_of(4)
+    for ch in (dict(n_group=7), dict(topk_group=9), dict(top_k=200, topk_group=1)):
+        bad = cfg_of(4, **ch)
+        assert gb.check_config(bad) == gb.EINVAL, ch
+    assert gb.check_config(c) == gb.OK
+
+
+class FakePtr:
+    """An aligned non-null address the library never dereferences here."""
+
+    def __init__(self, nbytes=1 << 20):
+        self.buf = ctypes.create_string_buffer(nbytes + 256)
+        self.addr = (ctypes.addressof(self.buf) + 255) & ~255
+        self.nbytes = nbytes
+
+    def data_ptr(self):
+        return self.addr
+
+    def numel(self):
+        return self.nbytes
+
+    def element_size(self):
+        return 1
+
+
+def test_entry_points_reject_bad_arguments_before_launching(lib):
+    c = cfg_of(1)
+    p = FakePtr()
+    small_ws = FakePtr(64)
+    with pytest.raises(gb.GbmoeError) as e:
+        gb.moe_route(c, None, p, None, None, p, p, p, stream=0)
+    assert e.value.status == gb.EINVAL
+    with pytest.raises(gb.GbmoeError) as e:
+        gb.moe_route(c, p, p, None, None, p, p, small_ws, stream=0)
+    assert e.value.status == gb.EWORKSPACE
+    with pytest.raises(gb.GbmoeError) as e:
+        gb.moe_permute(c, p, None, p, p, p, p, stream=0)
+    assert e.value.status == gb.EINVAL
+    w = gb.weights(p, None, p)
+    with pytest.raises(gb.GbmoeError) as e:
+        gb.moe_grouped_ffn(c, p, p, p, p, w, p, p, stream=0)
+    assert e.value.status == gb.EINVAL
+    with pytest.raises(gb.GbmoeError) as e:
+        gb.moe_shared_ffn(c, p, gb.weights(p, p, p), p, p, stream=0)  # config has no shared expert
+    assert e.value.status == gb.EINVAL
+    c4 = cfg_of(4)
+    with pytest.raises(gb.GbmoeError) as e:
+        gb.moe_forward(c4, p, p, None, None, gb.weights(p, p, p), gb.weights(p, p, p), p, p, stream=0)  # no fp8 scales
+    assert e.value.status == gb.EINVAL
+    assert gb.status_string(gb.EDEVICE_TIMEOUT) == "device-side wait timed out"

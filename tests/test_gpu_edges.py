@@ -1,0 +1,111 @@
+"""GPU parity on edge shapes: one token, no tokens, ragged tiles, every token
+on one expert, k = E, a single expert, and argument errors."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2607_12875_gb300 as gb
+import synth
+from gpu_helpers import act_np, config, rel_err, to_device, tol_for, wbundle, workspace
+
+pytestmark = pytest.mark.gpu
+
+TINY = synth.WORKLOADS[1]
+
+
+def run(wl, route, inp=None):
+    inp = synth.make_inputs(wl) if inp is None else inp
+    dev = to_device(wl, inp)
+    cfg = config(wl, route)
+    ws = workspace(cfg)
+    out = torch.empty((wl.T, wl.H), dtype=dev["x"].dtype, device="cuda")
+    ids = torch.empty((max(wl.T, 1), wl.top_k), dtype=torch.int32, device="cuda")
+    counts = torch.empty(wl.E, dtype=torch.int32, device="cuda")
+    gb.moe_forward(cfg, dev["x"], dev["w_router"], dev["logit_bias"], dev["select_bias"], wbundle(dev["experts"]),
+                   wbundle(dev["shared"]), out, ws, topk_ids=ids if wl.T else None,
+                   counts=counts if wl.T else None)
+    torch.cuda.synchronize()
+    return inp, out, ids, counts
+
+
+def check(wl, route, inp=None):
+    inp, out, ids, counts = run(wl, route, inp)
+    ref = oracle.forward(wl, inp)
+    assert np.array_equal(ids.cpu().numpy()[: wl.T], ref["topk_ids"])
+    assert np.array_equal(counts.cpu().numpy(), ref["counts"])
+    err = rel_err(act_np(out), ref["out"])
+    assert err <= tol_for(wl), f"rel err {err:.3e}"
+    return ref
+
+
+@pytest.mark.parametrize("route", ["simt", "stream"])
+@pytest.mark.parametrize("act", ["f32", "bf16"])
+def test_single_token(route, act):
+    wl = TINY.replace(T=1, act=act, wq=act, seed=21)
+    check(wl, route)
+
+
+def test_no_tokens_is_a_noop():
+    wl = TINY.replace(T=0)
+    cfg = config(wl)
+    ws = workspace(cfg)
+    dev = to_device(wl, synth.make_inputs(wl.replace(T=1)))
+    out = torch.empty((0, wl.H), dtype=torch.float32, device="cuda")
+    gb.moe_forward(cfg, dev["x"], dev["w_router"], None, None, wbundle(dev["experts"]), None, out, ws)
+    torch.cuda.synchronize()
+
+
+@pytest.mark.parametrize("route", ["simt", "stream"])
+def test_ragged_tiles(route):
+    # 37 tokens x top-3 over 5 experts: no expert's row count is a tile multiple
+    wl = TINY.replace(T=37, E=5, top_k=3, act="bf16", wq="bf16", seed=22, H=512, I=256)
+    check(wl, route)
+
+
+@pytest.mark.parametrize("route", ["simt", "stream"])
+def test_every_token_on_one_expert(route):
+    wl = TINY.replace(T=70, E=8, top_k=2, seed=23, act="bf16", wq="bf16")
+    inp = synth.make_inputs(wl)
+    bias = np.zeros(wl.E, np.float32)
+    bias[5] = 1000.0
+    inp["logit_bias"] = bias
+    ref = check(wl, route, inp)
+    assert ref["counts"][5] == wl.T
+
+
+@pytest.mark.parametrize("route", ["simt", "stream"])
+def test_k_equals_E_and_single_expert(route):
+    check(TINY.replace(T=9, E=8, top_k=8, seed=24), route)
+    check(TINY.replace(T=9, E=1, top_k=1, seed=25), route)
+
+
+@pytest.mark.parametrize("wq", ["fp8_b128", "int4_g128"])
+@pytest.mark.parametrize("route", ["simt", "stream"])
+def test_quantised_weights_small(wq, route):
+    wl = TINY.replace(T=24, E=4, top_k=2, act="bf16", wq=wq, H=256, I=256, seed=26)
+    check(wl, route)
+
+
+def test_sigmoid_grouped_small_with_shared():
+    wl = TINY.replace(T=40, E=16, top_k=4, act="bf16", wq="fp8_b128", H=256, I=128, seed=27, score="sigmoid",
+                      routed_scale=2.5, n_group=4, topk_group=2, has_shared=True, I_shared=256,
+                      select_bias_sigma=0.01)
+    check(wl, "simt")
+    check(wl, "stream")
+
+
+def test_argument_errors_launch_nothing():
+    wl = TINY
+    cfg = config(wl)
+    ws = workspace(cfg)
+    x = torch.zeros((wl.T, wl.H), device="cuda")
+    wr = torch.zeros((wl.E, wl.H), device="cuda")
+    ids = torch.empty((wl.T, wl.top_k), dtype=torch.int32, device="cuda")
+    w = torch.empty((wl.T, wl.top_k), dtype=torch.float32, device="cuda")
+    with pytest.raises(gb.GbmoeError) as e:
+        gb.moe_route(cfg, x, wr, None, None, ids, w, ws[: gb.workspace_size(cfg) // 4])
+    assert e.value.status == gb.EWORKSPACE
+    with pytest.raises(gb.GbmoeError) as e:
+        gb.moe_route(cfg, x[:, 1:], wr, None, None, ids, w, ws)  # misaligned x
+    assert e.value.status == gb.EINVAL
