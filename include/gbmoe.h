@@ -211,6 +211,25 @@ int moe_forward_hostio(const gbmoe_config* cfg, const void* x_host, const void* 
  */
 int moe_device_status(void* workspace, void* stream, int32_t* status);
 
+/*
+ * moe_permute without a workspace: the same grouping as moe_permute (same
+ * outputs, bit for bit), with its scratch held in a static device array
+ * inside this library instead of a caller buffer. The paper has no
+ * counterpart; this exists for callers that cannot allocate device memory
+ * for a call: plain C hosts with no device allocator of their own, serving
+ * engines that reserve all device memory up front and lend out no scratch,
+ * and code that runs where cudaMalloc is not allowed. The array is 1 MiB
+ * (262144 int32) per device, held by every GPU that loads the library until
+ * the process exits; problems needing more, 2 * ceil(T*k / 1024) * E ints,
+ * return GBMOE_EUNSUPPORTED without launching anything. The call allocates
+ * nothing. Its first call on each device looks up the array's device
+ * address (cudaGetSymbolAddress, with that device current), so make that
+ * first call before any stream capture. All calls share the array: calls
+ * that overlap on the GPU (unordered streams) race; order them.
+ */
+int moe_permute_noalloc(const gbmoe_config* cfg, const int32_t* topk_ids, int32_t* counts, int32_t* offsets,
+                        int32_t* sorted_pair, int32_t* pair_pos, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -27,7 +27,7 @@ ROUTES = {"auto": FFN_AUTO, "stream": FFN_STREAM, "simt": FFN_SIMT, "tc": FFN_TC
 # every function include/gbmoe.h declares
 EXPORTS = ("gbmoe_status_string", "gbmoe_check_config", "gbmoe_workspace_size", "moe_route", "moe_permute",
            "moe_grouped_ffn", "moe_shared_ffn", "moe_combine", "moe_forward", "moe_forward_hostio",
-           "moe_device_status")
+           "moe_device_status", "moe_permute_noalloc")
 
 
 class GbmoeError(RuntimeError):
@@ -75,6 +75,7 @@ def lib() -> ctypes.CDLL:
         L.moe_forward.argtypes = [cfgp, vp, vp, fp, fp, wp, wp, vp, vp, vp, vp, vp, sz, vp]
         L.moe_forward_hostio.argtypes = [cfgp, vp, vp, fp, fp, wp, wp, vp, vp, sz, vp]
         L.moe_device_status.argtypes = [vp, vp, i32p]
+        L.moe_permute_noalloc.argtypes = [cfgp, vp, vp, vp, vp, vp, vp]
         _lib = L
     return _lib
 
@@ -170,3 +171,9 @@ def moe_device_status(ws, stream=None) -> int:
     st = ctypes.c_int32(0)
     _check(lib().moe_device_status(_ptr(ws), _stream(stream), ctypes.byref(st)), "moe_device_status")
     return st.value
+
+
+def moe_permute_noalloc(cfg, topk_ids, counts, offsets, sorted_pair, pair_pos, stream=None):
+    """moe_permute with the library's static scratch instead of a workspace."""
+    _check(lib().moe_permute_noalloc(ctypes.byref(cfg), _ptr(topk_ids), _ptr(counts), _ptr(offsets),
+                                     _ptr(sorted_pair), _ptr(pair_pos), _stream(stream)), "moe_permute_noalloc")
