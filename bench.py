@@ -36,6 +36,11 @@ import synth  # noqa: E402
 METRIC = "MoE layer tokens/sec at 1 GB300; % of HBM (decode) / tensor-core (prefill) roofline"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
+# DRAM bytes per launch of the dominant kernel(s) from one ncu capture
+# (dram__bytes_read.sum + dram__bytes_write.sum), keyed by (workload, route);
+# absent (null) whenever the kernel changed since the counters were taken.
+TRAFFIC: dict = {}
+
 
 def peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
@@ -304,12 +309,22 @@ def main():
     torch.cuda.synchronize()
     ffn_ms = fs.elapsed_time(fe) / args.steps
     pk, pk_kind = peaks()
-    routed_bytes = algorithmic_weight_bytes(wl.replace(has_shared=False), active)
-    achieved = routed_bytes / (ffn_ms / 1e3) / 1e9
-    roofline = {"bound": "hbm", "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s",
-                "frac": achieved / pk["hbm_gbs"], "traffic": None, "peak_kind": pk_kind,
-                "kernel": "moe_grouped_ffn (weight-streaming route: gate/up + down)",
-                "algorithmic_bytes": routed_bytes, "active_experts": active, "ms_per_launch": ffn_ms}
+    route = gb.ffn_route(cfg)
+    if route == "stream":
+        routed_bytes = algorithmic_weight_bytes(wl.replace(has_shared=False), active)
+        achieved = routed_bytes / (ffn_ms / 1e3) / 1e9
+        roofline = {"bound": "hbm", "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s",
+                    "frac": achieved / pk["hbm_gbs"], "traffic": TRAFFIC.get((wl.name, route)),
+                    "peak_kind": pk_kind, "kernel": "moe_grouped_ffn, weight-streaming route (gate/up + down)",
+                    "algorithmic_bytes": routed_bytes, "active_experts": active, "ms_per_launch": ffn_ms}
+    else:
+        flops = 6.0 * wl.P * wl.H * wl.I
+        achieved = flops / (ffn_ms / 1e3) / 1e12
+        roofline = {"bound": "tensor", "achieved": achieved, "peak": pk["bf16_tflops"], "unit": "TFLOP/s",
+                    "frac": achieved / pk["bf16_tflops"], "traffic": TRAFFIC.get((wl.name, route)),
+                    "peak_kind": f"{pk_kind} bf16 dense burst", "kernel": f"moe_grouped_ffn, {route} route "
+                    "(gather + gate/up GEMM with SwiGLU + down GEMM)", "algorithmic_flops": flops,
+                    "active_experts": active, "ms_per_launch": ffn_ms}
 
     # end to end through the public host-buffer entry point
     x_host = x.cpu().pin_memory()
@@ -333,8 +348,9 @@ def main():
            "d2h_bytes_per_step": io_bytes}
 
     # kernels this library launched per step: gate logits + expert choice, 3 for the
-    # permutation, schedule + 2 per expert-FFN problem, combine
-    per_step = 2 + 3 + 3 + (3 if wl.has_shared else 0) + 1
+    # permutation, per FFN problem a schedule kernel + 2 (+ a row gather for the routed experts on the
+    # tensor-core route), combine
+    per_step = 2 + 3 + (4 if route == "tc" else 3) + (3 if wl.has_shared else 0) + 1
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

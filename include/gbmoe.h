@@ -114,6 +114,11 @@ int gbmoe_check_config(const gbmoe_config* cfg);
  * other calls need no more). 0 if the config is invalid. */
 size_t gbmoe_workspace_size(const gbmoe_config* cfg);
 
+/* The FFN route (GBMOE_FFN_STREAM, _SIMT or _TC) that moe_forward runs for
+ * cfg: for the routed experts (shared = 0) or the shared expert (shared = 1).
+ * Negative status if the config is invalid. */
+int gbmoe_ffn_route(const gbmoe_config* cfg, int shared);
+
 /*
  * MoE Gate (Fig. 1 and Fig. 3). For every token t:
  *   l[t,e] = x[t,:] . w_router[e,:] (+ logit_bias[e]), fp32, in a fixed order:

@@ -25,7 +25,8 @@ DTYPES = {"f32": F32, "bf16": BF16, "fp8_b128": FP8_E4M3_B128, "int4_g128": INT4
 ROUTES = {"auto": FFN_AUTO, "stream": FFN_STREAM, "simt": FFN_SIMT, "tc": FFN_TC}
 
 # every function include/gbmoe.h declares
-EXPORTS = ("gbmoe_status_string", "gbmoe_check_config", "gbmoe_workspace_size", "moe_route", "moe_permute",
+EXPORTS = ("gbmoe_status_string", "gbmoe_check_config", "gbmoe_workspace_size", "gbmoe_ffn_route", "moe_route",
+           "moe_permute",
            "moe_grouped_ffn", "moe_shared_ffn", "moe_combine", "moe_forward", "moe_forward_hostio",
            "moe_device_status", "moe_permute_noalloc")
 
@@ -67,6 +68,7 @@ def lib() -> ctypes.CDLL:
         L.gbmoe_check_config.argtypes = [cfgp]
         L.gbmoe_workspace_size.argtypes = [cfgp]
         L.gbmoe_workspace_size.restype = sz
+        L.gbmoe_ffn_route.argtypes = [cfgp, ctypes.c_int]
         L.moe_route.argtypes = [cfgp, vp, vp, fp, fp, vp, vp, vp, sz, vp]
         L.moe_permute.argtypes = [cfgp, vp, vp, vp, vp, vp, vp, sz, vp]
         L.moe_grouped_ffn.argtypes = [cfgp, vp, vp, vp, vp, wp, vp, vp, sz, vp]
@@ -121,6 +123,14 @@ def check_config(cfg: Config) -> int:
 
 def workspace_size(cfg: Config) -> int:
     return lib().gbmoe_workspace_size(ctypes.byref(cfg))
+
+
+def ffn_route(cfg: Config, shared: bool = False) -> str:
+    """Name of the FFN route moe_forward runs for cfg ("stream", "simt", "tc")."""
+    r = lib().gbmoe_ffn_route(ctypes.byref(cfg), int(bool(shared)))
+    if r < 0:
+        raise GbmoeError(r, "gbmoe_ffn_route")
+    return {FFN_STREAM: "stream", FFN_SIMT: "simt", FFN_TC: "tc"}[r]
 
 
 def moe_route(cfg, x, w_router, logit_bias, select_bias, topk_ids, topk_w, ws, stream=None):

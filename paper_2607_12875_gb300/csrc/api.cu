@@ -16,7 +16,6 @@ namespace {
 constexpr size_t kAlign = 256;
 constexpr int kStreamRowsPerPass = 8;       // matches the streaming kernels' pass height
 constexpr size_t kSmemBudget = 227 * 1024;  // per-CTA shared memory on sm_103a
-constexpr bool kAutoTensorCores = false;    // AUTO picks the tensor-core route once it is validated
 
 size_t align_up(size_t v) { return (v + kAlign - 1) & ~(kAlign - 1); }
 
@@ -62,7 +61,7 @@ int pick_route(const gbmoe_config* c, int64_t n_rows, int E, int I) {
     int r = c->ffn_route;
     if (r != GBMOE_FFN_AUTO) return r;
     if (n_rows <= 16 * (int64_t)E && stream_fits(c->H, I, c->act_dtype)) return GBMOE_FFN_STREAM;
-    if (c->act_dtype == GBMOE_BF16 && kAutoTensorCores) {
+    if (c->act_dtype == GBMOE_BF16) {
         FfnProblem probe{};
         probe.act_dtype = c->act_dtype;
         probe.w_dtype = c->w_dtype;
@@ -205,6 +204,13 @@ int gbmoe_check_config(const gbmoe_config* cfg) { return check_cfg(cfg); }
 size_t gbmoe_workspace_size(const gbmoe_config* cfg) {
     if (check_cfg(cfg) != GBMOE_OK) return 0;
     return layout(cfg).total;
+}
+
+int gbmoe_ffn_route(const gbmoe_config* cfg, int shared) {
+    int s = check_cfg(cfg);
+    if (s) return s;
+    if (shared) return cfg->has_shared ? pick_route(cfg, cfg->T, 1, cfg->I_shared) : GBMOE_EINVAL;
+    return pick_route(cfg, (int64_t)cfg->T * cfg->top_k, cfg->E, cfg->I);
 }
 
 int moe_route(const gbmoe_config* cfg, const void* x, const void* w_router, const float* logit_bias,

@@ -19,10 +19,18 @@
 //             h = silu(gate) * up for the gate/up GEMM (B rows 0-127 are the
 //             gate rows, 128-255 the up rows of the same 128 columns), plain
 //             y for the down GEMM.
+// Quantised weights (fp8 e4m3 with 128x128 block scales, int4 with 128-wide
+// group scales) take the same path with eight more warps: TMA brings the raw
+// weight tile (64- or 32-byte swizzled rows) next to the A tile, and
+// warps 6-13, one B row per thread, decode it, apply the scale and write
+// the bf16 operand in the 128-byte-swizzled layout the MMA reads, then
+// signal the MMA warp. Decoding inside the kernel means no dequantised copy
+// of the weights ever exists in HBM.
 // Every mbarrier wait is bounded (about two seconds); on expiry the CTA sets
 // the device error word, stops issuing work, drains what it issued and
 // frees its TMEM.
 #include <cuda.h>
+#include <cuda_fp16.h>
 
 #include "common.cuh"
 #include "ffn_sched.h"
@@ -32,15 +40,37 @@ namespace gbmoe {
 namespace tc {
 
 constexpr int BM = 128, BN = 256, BK = 64;  // BK bf16 = 128 bytes = one swizzle row
-constexpr int STAGES = 4;
 constexpr int A_BYTES = BM * BK * 2;
 constexpr int B_BYTES = BN * BK * 2;
-constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int TMEM_COLS = 512;
-constexpr int NUM_THREADS = 192;
-constexpr int NUM_BARS = 2 * STAGES + 4 + 1;
-constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + NUM_BARS * 8 + 16;
+constexpr int CONVERT_WARPS = 8;  // one thread per B row (BN = 256)
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;
+
+// Per weight format: bytes of the raw B tile TMA brings in (0 = B is loaded
+// as bf16 directly), pipeline depth, threads.
+template <int WQ>
+struct Fmt;
+template <>
+struct Fmt<GBMOE_BF16> {
+    static constexpr int RAW_BYTES = 0, STAGES = 4, THREADS = 192;
+};
+template <>
+struct Fmt<GBMOE_FP8_E4M3_B128> {
+    static constexpr int RAW_BYTES = BN * BK, STAGES = 3, THREADS = 192 + CONVERT_WARPS * 32;
+};
+template <>
+struct Fmt<GBMOE_INT4_G128> {
+    static constexpr int RAW_BYTES = BN * BK / 2, STAGES = 4, THREADS = 192 + CONVERT_WARPS * 32;
+};
+
+template <int WQ>
+struct Layout {
+    static constexpr int STAGES = Fmt<WQ>::STAGES;
+    static constexpr int STAGE_BYTES = A_BYTES + B_BYTES + Fmt<WQ>::RAW_BYTES;
+    static constexpr int NUM_BARS = 3 * STAGES + 4 + 1;
+    static constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + NUM_BARS * 8 + 16;
+    static_assert(SMEM_BYTES <= 232448, "shared memory per CTA");
+};
 
 struct Params {
     int K;                 // reduction length
@@ -55,6 +85,8 @@ struct Params {
     int64_t n_rows;
     __nv_bfloat16* out;
     int32_t* err;
+    const void* scale0;  // scales of the B rows in the first / second half of the tile
+    const void* scale1;
 };
 
 // ------------------------------------------------------------ PTX wrappers
@@ -183,6 +215,57 @@ __device__ __forceinline__ void store_bf16x32(__nv_bfloat16* dst, const float (&
     }
 }
 
+// ----------------------------------------------------- weight decoding
+
+// 16-byte chunk c (0..7) of row r of a 128-byte-swizzled tile
+__device__ __forceinline__ uint32_t sw128_off(int r, int c) { return (uint32_t)(r * 128 + ((c ^ (r & 7)) << 4)); }
+// same for rows of 64 bytes (chunks 0..3) and 32 bytes (chunks 0..1) as TMA
+// writes them with 64- and 32-byte swizzling
+__device__ __forceinline__ uint32_t sw64_off(int r, int c) { return (uint32_t)(r * 64 + ((c ^ ((r >> 1) & 3)) << 4)); }
+__device__ __forceinline__ uint32_t sw32_off(int r, int c) { return (uint32_t)(r * 32 + ((c ^ ((r >> 2) & 1)) << 4)); }
+
+// two e4m3 values (low byte = first element) -> two fp32
+__device__ __forceinline__ float2 e4m3x2_to_f32x2(uint32_t two_bytes) {
+    uint32_t h2;
+    asm("cvt.rn.f16x2.e4m3x2 %0, %1;" : "=r"(h2) : "h"((unsigned short)two_bytes));
+    __half2 h = *reinterpret_cast<__half2*>(&h2);
+    return __half22float2(h);
+}
+
+// 16 e4m3 weights (one 16-byte raw chunk) times the block scale -> 16 bf16 in two 16-byte chunks
+__device__ __forceinline__ void decode_fp8_16(const uint4 raw, float sc, uint4& o0, uint4& o1) {
+    const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
+    uint32_t packed[8];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        float2 a = e4m3x2_to_f32x2(w[i] & 0xffffu);
+        float2 b = e4m3x2_to_f32x2(w[i] >> 16);
+        packed[2 * i] = pack_bf16x2(a.x * sc, a.y * sc);
+        packed[2 * i + 1] = pack_bf16x2(b.x * sc, b.y * sc);
+    }
+    o0 = make_uint4(packed[0], packed[1], packed[2], packed[3]);
+    o1 = make_uint4(packed[4], packed[5], packed[6], packed[7]);
+}
+
+// 8 int4 weights (one 32-bit word, element 0 in the low nibble) times the
+// group scale -> 8 bf16 (one 16-byte chunk). A nibble v becomes the bf16
+// 128 + (v xor 8) by OR-ing it into the mantissa of 128.0, and 136 is
+// subtracted exactly, which leaves the two's-complement value; then one bf16
+// multiply by the scale.
+__device__ __forceinline__ uint4 decode_int4_8(uint32_t w, __nv_bfloat162 sc2) {
+    const __nv_bfloat162 k136 = __floats2bfloat162_rn(136.0f, 136.0f);
+    uint32_t p[4];  // p[i] holds elements (i, i + 4)
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        uint32_t t = ((w >> (4 * i)) & 0x000f000fu) ^ 0x43084308u;
+        __nv_bfloat162 v = *reinterpret_cast<__nv_bfloat162*>(&t);
+        v = __hmul2(__hsub2(v, k136), sc2);
+        p[i] = *reinterpret_cast<uint32_t*>(&v);
+    }
+    return make_uint4(__byte_perm(p[0], p[1], 0x5410), __byte_perm(p[2], p[3], 0x5410),
+                      __byte_perm(p[0], p[1], 0x7632), __byte_perm(p[2], p[3], 0x7632));
+}
+
 // ------------------------------------------------------------------ kernel
 
 struct Work {
@@ -205,20 +288,32 @@ __device__ __forceinline__ Work decode_work(const Params& p, int w) {
     return r;
 }
 
-__global__ void __launch_bounds__(NUM_THREADS, 1)
+// first B row (in the stacked [E * rows_per_expert, K] tensor) of each tile half
+__device__ __forceinline__ void b_rows(const Params& p, const Work& wk, int& b0, int& b1) {
+    b0 = wk.e * p.b_rows_per_expert + (p.swiglu ? wk.nt * (BN / 2) : wk.nt * BN);
+    b1 = p.swiglu ? b0 : b0 + BN / 2;
+}
+
+template <int WQ>
+__global__ void __launch_bounds__(Fmt<WQ>::THREADS, 1)
 tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b0,
                const __grid_constant__ CUtensorMap tm_b1, const Params p) {
+    using L = Layout<WQ>;
+    constexpr int STAGES = L::STAGES;
+    constexpr int RAW = Fmt<WQ>::RAW_BYTES;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
     uint8_t* sA = smem;
     uint8_t* sB = smem + STAGES * A_BYTES;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
-    uint64_t* full = bars;
-    uint64_t* empty = bars + STAGES;
-    uint64_t* tfull = bars + 2 * STAGES;
-    uint64_t* tempty = bars + 2 * STAGES + 2;
-    uint64_t* drain = bars + 2 * STAGES + 4;
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + NUM_BARS);
+    uint8_t* sR = smem + STAGES * (A_BYTES + B_BYTES);  // raw quantised B tiles
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * L::STAGE_BYTES);
+    uint64_t* full = bars;                 // TMA landed (A + B or A + raw B)
+    uint64_t* empty = bars + STAGES;       // MMAs reading the slot finished
+    uint64_t* conv = bars + 2 * STAGES;    // bf16 B written by the converters
+    uint64_t* tfull = bars + 3 * STAGES;
+    uint64_t* tempty = bars + 3 * STAGES + 2;
+    uint64_t* drain = bars + 3 * STAGES + 4;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + L::NUM_BARS);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -226,6 +321,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(&full[s], 1);
             mbar_init(&empty[s], 1);
+            mbar_init(&conv[s], CONVERT_WARPS);
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(&tfull[a], 1);
@@ -257,15 +353,22 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
         bool ok = true;
         for (int w = blockIdx.x; w < total && ok; w += gridDim.x) {
             const Work wk = decode_work(p, w);
-            const int b0 = wk.e * p.b_rows_per_expert + (p.swiglu ? wk.nt * (BN / 2) : wk.nt * BN);
-            const int b1 = p.swiglu ? b0 : b0 + BN / 2;
+            int b0, b1;
+            b_rows(p, wk, b0, b1);
             for (int kb = 0; kb < nkb; ++kb) {
                 if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, p.err)) { ok = false; break; }
                 inflight &= ~(1u << stage);
-                mbar_expect_tx(&full[stage], STAGE_BYTES);
+                mbar_expect_tx(&full[stage], A_BYTES + (RAW ? RAW : B_BYTES));
                 tma_load_2d(sA + stage * A_BYTES, &tm_a, kb * BK, (int)wk.row0, &full[stage]);
-                tma_load_2d(sB + stage * B_BYTES, &tm_b0, kb * BK, b0, &full[stage]);
-                tma_load_2d(sB + stage * B_BYTES + B_BYTES / 2, &tm_b1, kb * BK, b1, &full[stage]);
+                if (RAW == 0) {
+                    tma_load_2d(sB + stage * B_BYTES, &tm_b0, kb * BK, b0, &full[stage]);
+                    tma_load_2d(sB + stage * B_BYTES + B_BYTES / 2, &tm_b1, kb * BK, b1, &full[stage]);
+                } else {
+                    // raw boxes are BK elements wide: BK bytes (fp8) or BK/2 bytes (int4)
+                    const int x = (WQ == GBMOE_INT4_G128) ? kb * (BK / 2) : kb * BK;
+                    tma_load_2d(sR + stage * RAW, &tm_b0, x, b0, &full[stage]);
+                    tma_load_2d(sR + stage * RAW + RAW / 2, &tm_b1, x, b1, &full[stage]);
+                }
                 inflight |= 1u << stage;
                 inflight_par = (inflight_par & ~(1u << stage)) | (phase << stage);
                 if (++stage == STAGES) { stage = 0; phase ^= 1; }
@@ -294,6 +397,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
             const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
             for (int kb = 0; kb < nkb; ++kb) {
                 if (!mbar_wait(&full[stage], phase, abort_flag, p.err)) { ok = false; break; }
+                if (RAW && !mbar_wait(&conv[stage], phase, abort_flag, p.err)) { ok = false; break; }
                 tc_fence_after();
                 const uint64_t da = sw128_desc(smem_u32(sA + stage * A_BYTES));
                 const uint64_t db = sw128_desc(smem_u32(sB + stage * B_BYTES));
@@ -315,9 +419,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
             while (!mbar_try_wait(drain, 0) && global_ns() - t0 < kWaitLimitNs) {
             }
         }
-    } else if (warp >= 2) {
+    } else if (warp >= 2 && warp < 6) {
         // -------------------------------------------------------- epilogue
-        const int q = warp & 3;  // TMEM lane quarter of this warp
+        const int q = warp & 3;       // TMEM lane quarter of this warp
         const int r = q * 32 + lane;  // tile row of this thread
         int acc = 0;
         uint32_t acc_phase = 0;
@@ -351,6 +455,53 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
             tc_fence_before();
             mbar_arrive(&tempty[acc]);
             if (++acc == 2) { acc = 0; acc_phase ^= 1; }
+        }
+    } else if (RAW && warp >= 6) {
+        // ------------------------------------------- weight decode (B rows)
+        const int r = threadIdx.x - 6 * 32;  // B row 0..255 of the tile
+        const int half = r >> 7;
+        const void* scales = half ? p.scale1 : p.scale0;
+        const int kgroups = p.K / 128;
+        int stage = 0;
+        uint32_t phase = 0;
+        bool ok = true;
+        for (int w = blockIdx.x; w < total && ok; w += gridDim.x) {
+            const Work wk = decode_work(p, w);
+            int b0, b1;
+            b_rows(p, wk, b0, b1);
+            const int64_t brow = (half ? b1 : b0) + (r & 127);  // absolute row of the stacked B tensor
+            for (int kb = 0; kb < nkb; ++kb) {
+                if (!mbar_wait(&full[stage], phase, abort_flag, p.err)) { ok = false; break; }
+                const uint8_t* raw = sR + stage * RAW;
+                uint8_t* dstB = sB + stage * B_BYTES;
+                if (WQ == GBMOE_FP8_E4M3_B128) {
+                    const float sc = static_cast<const float*>(scales)[(brow / 128) * kgroups + kb / 2];
+#pragma unroll
+                    for (int c = 0; c < 4; ++c) {
+                        const uint4 v = *reinterpret_cast<const uint4*>(raw + sw64_off(r, c));
+                        uint4 o0, o1;
+                        decode_fp8_16(v, sc, o0, o1);
+                        *reinterpret_cast<uint4*>(dstB + sw128_off(r, 2 * c)) = o0;
+                        *reinterpret_cast<uint4*>(dstB + sw128_off(r, 2 * c + 1)) = o1;
+                    }
+                } else {
+                    const __nv_bfloat16 sb = static_cast<const __nv_bfloat16*>(scales)[brow * kgroups + kb / 2];
+                    const __nv_bfloat162 sc2 = __halves2bfloat162(sb, sb);
+#pragma unroll
+                    for (int c = 0; c < 2; ++c) {
+                        const uint4 v = *reinterpret_cast<const uint4*>(raw + sw32_off(r, c));
+                        const uint32_t ws[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+                        for (int i = 0; i < 4; ++i)
+                            *reinterpret_cast<uint4*>(dstB + sw128_off(r, 4 * c + i)) = decode_int4_8(ws[i], sc2);
+                    }
+                }
+                // make the generic-proxy writes visible to the tensor core, then signal
+                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&conv[stage]);
+                if (++stage == STAGES) { stage = 0; phase ^= 1; }
+            }
         }
     }
     tc_fence_before();
@@ -397,17 +548,34 @@ static EncodeTiled encode_fn() {
     return fn;
 }
 
-// bf16 matrix [rows, cols] row-major; boxes of 64 columns x 128 rows, 128-byte swizzle
-static bool make_map(CUtensorMap* m, const void* base, int64_t rows, int64_t cols) {
+// 2-D row-major matrix [rows, row_bytes / elem] in boxes of box_x elements x
+// 128 rows with the given swizzle
+static bool make_map(CUtensorMap* m, const void* base, int64_t rows, int64_t row_bytes, CUtensorMapDataType dt,
+                     int elem_bytes, int box_x, CUtensorMapSwizzle sw) {
     EncodeTiled fn = encode_fn();
     if (!fn) return false;
-    cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
-    cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
-    cuuint32_t box[2] = {BK, 128};
+    cuuint64_t dims[2] = {(cuuint64_t)(row_bytes / elem_bytes), (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)row_bytes};
+    cuuint32_t box[2] = {(cuuint32_t)box_x, 128};
     cuuint32_t estr[2] = {1, 1};
-    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
-              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+    return fn(m, dt, 2, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+static bool map_bf16(CUtensorMap* m, const void* base, int64_t rows, int64_t cols) {
+    return make_map(m, base, rows, cols * 2, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, BK, CU_TENSOR_MAP_SWIZZLE_128B);
+}
+
+// B operand [rows, K] in the weight format WQ
+static bool map_weights(CUtensorMap* m, int wq, const void* base, int64_t rows, int64_t K) {
+    switch (wq) {
+        case GBMOE_BF16: return map_bf16(m, base, rows, K);
+        case GBMOE_FP8_E4M3_B128:
+            return make_map(m, base, rows, K, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, BK, CU_TENSOR_MAP_SWIZZLE_64B);
+        case GBMOE_INT4_G128:
+            return make_map(m, base, rows, K / 2, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, BK / 2, CU_TENSOR_MAP_SWIZZLE_32B);
+        default: return false;
+    }
 }
 
 static int num_sms() {
@@ -417,25 +585,33 @@ static int num_sms() {
     return n > 0 ? n : 1;
 }
 
-static cudaError_t launch_gemm(const CUtensorMap& a, const CUtensorMap& b0, const CUtensorMap& b1, const Params& prm,
-                               int64_t max_work, cudaStream_t stream) {
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(tc_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
-        if (e != cudaSuccess) return e;
-        attr_set = true;
-    }
+template <int WQ>
+static cudaError_t launch_gemm_t(const CUtensorMap& a, const CUtensorMap& b0, const CUtensorMap& b1,
+                                 const Params& prm, int64_t max_work, cudaStream_t stream) {
+    cudaError_t e = cudaFuncSetAttribute(tc_gemm_kernel<WQ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         Layout<WQ>::SMEM_BYTES);
+    if (e != cudaSuccess) return e;
     const int grid = (int)min64(num_sms(), max_work);
     if (grid <= 0) return cudaSuccess;
-    tc_gemm_kernel<<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(a, b0, b1, prm);
+    tc_gemm_kernel<WQ><<<grid, Fmt<WQ>::THREADS, Layout<WQ>::SMEM_BYTES, stream>>>(a, b0, b1, prm);
     return cudaGetLastError();
+}
+
+static cudaError_t launch_gemm(int wq, const CUtensorMap& a, const CUtensorMap& b0, const CUtensorMap& b1,
+                               const Params& prm, int64_t max_work, cudaStream_t stream) {
+    switch (wq) {
+        case GBMOE_BF16: return launch_gemm_t<GBMOE_BF16>(a, b0, b1, prm, max_work, stream);
+        case GBMOE_FP8_E4M3_B128: return launch_gemm_t<GBMOE_FP8_E4M3_B128>(a, b0, b1, prm, max_work, stream);
+        case GBMOE_INT4_G128: return launch_gemm_t<GBMOE_INT4_G128>(a, b0, b1, prm, max_work, stream);
+        default: return cudaErrorInvalidValue;
+    }
 }
 
 }  // namespace tc
 
 bool ffn_tc_supported(const FfnProblem& p) {
-    return p.act_dtype == GBMOE_BF16 && p.w_dtype == GBMOE_BF16 && p.H % 256 == 0 && p.I % 128 == 0 &&
-           tc::encode_fn() != nullptr;
+    const bool wq_ok = p.w_dtype == GBMOE_BF16 || p.w_dtype == GBMOE_FP8_E4M3_B128 || p.w_dtype == GBMOE_INT4_G128;
+    return p.act_dtype == GBMOE_BF16 && wq_ok && p.H % 256 == 0 && p.I % 128 == 0 && tc::encode_fn() != nullptr;
 }
 
 cudaError_t launch_ffn_tc(const FfnProblem& p, cudaStream_t stream) {
@@ -443,31 +619,38 @@ cudaError_t launch_ffn_tc(const FfnProblem& p, cudaStream_t stream) {
     if (p.n_rows == 0) return cudaSuccess;
     cudaError_t err = launch_ffn_schedule(p.counts, p.E, p.n_rows, BM, p.sched, stream);
     if (err != cudaSuccess) return err;
-    // x rows in sorted order
-    const int vpr = p.H * 2 / 16;
-    const int64_t nvec = p.n_rows * vpr;
-    const int gblocks = (int)min64((nvec + 255) / 256, 152 * 16);
-    gather_rows_kernel<<<gblocks, 256, 0, stream>>>(static_cast<const uint4*>(p.x), p.sorted_pair, p.pair_div,
-                                                    p.n_rows, vpr, static_cast<uint4*>(p.x_sorted));
-    if ((err = cudaGetLastError()) != cudaSuccess) return err;
+    // A operand of the gate/up GEMM: x rows in sorted order (a gathered copy),
+    // or x itself when rows are already in order (no sorted_pair: shared expert)
+    const void* a_rows = p.x;
+    if (p.sorted_pair) {
+        const int vpr = p.H * 2 / 16;
+        const int64_t nvec = p.n_rows * vpr;
+        const int gblocks = (int)min64((nvec + 255) / 256, 152 * 16);
+        gather_rows_kernel<<<gblocks, 256, 0, stream>>>(static_cast<const uint4*>(p.x), p.sorted_pair, p.pair_div,
+                                                        p.n_rows, vpr, static_cast<uint4*>(p.x_sorted));
+        if ((err = cudaGetLastError()) != cudaSuccess) return err;
+        a_rows = p.x_sorted;
+    }
 
     const int64_t max_m = sched_max_tiles(p.E, p.n_rows, BM);
     CUtensorMap ma, mg, mu, mh, md;
-    if (!make_map(&ma, p.x_sorted, p.n_rows, p.H) || !make_map(&mg, p.w_gate, (int64_t)p.E * p.I, p.H) ||
-        !make_map(&mu, p.w_up, (int64_t)p.E * p.I, p.H) || !make_map(&mh, p.h, p.n_rows, p.I) ||
-        !make_map(&md, p.w_down, (int64_t)p.E * p.H, p.I))
+    if (!map_bf16(&ma, a_rows, p.n_rows, p.H) || !map_weights(&mg, p.w_dtype, p.w_gate, (int64_t)p.E * p.I, p.H) ||
+        !map_weights(&mu, p.w_dtype, p.w_up, (int64_t)p.E * p.I, p.H) || !map_bf16(&mh, p.h, p.n_rows, p.I) ||
+        !map_weights(&md, p.w_dtype, p.w_down, (int64_t)p.E * p.H, p.I))
         return cudaErrorInvalidValue;
 
     Params g{};
     g.K = p.H; g.n_tiles = p.I / (BN / 2); g.out_cols = p.I; g.b_rows_per_expert = p.I; g.swiglu = 1;
     g.counts = p.counts; g.offsets = p.offsets; g.sched = p.sched; g.E = p.E; g.n_rows = p.n_rows;
     g.out = static_cast<__nv_bfloat16*>(p.h); g.err = p.err;
-    if ((err = launch_gemm(ma, mg, mu, g, max_m * g.n_tiles, stream)) != cudaSuccess) return err;
+    g.scale0 = p.s_gate; g.scale1 = p.s_up;
+    if ((err = launch_gemm(p.w_dtype, ma, mg, mu, g, max_m * g.n_tiles, stream)) != cudaSuccess) return err;
 
     Params d = g;
     d.K = p.I; d.n_tiles = p.H / BN; d.out_cols = p.H; d.b_rows_per_expert = p.H; d.swiglu = 0;
     d.out = static_cast<__nv_bfloat16*>(p.y);
-    return launch_gemm(mh, md, md, d, max_m * d.n_tiles, stream);
+    d.scale0 = p.s_down; d.scale1 = p.s_down;
+    return launch_gemm(p.w_dtype, mh, md, md, d, max_m * d.n_tiles, stream);
 }
 
 }  // namespace gbmoe

@@ -26,9 +26,10 @@ def forward(wl, dev, route):
     return out, ids
 
 
+@pytest.mark.parametrize("wq", ["bf16", "fp8_b128", "int4_g128"])
 @pytest.mark.parametrize("T,E,k,H,I", [(200, 4, 2, 512, 256), (1000, 4, 2, 256, 384), (333, 16, 3, 768, 128)])
-def test_tc_small_ragged(T, E, k, H, I):
-    wl = BASE.replace(T=T, E=E, top_k=k, H=H, I=I, seed=T + E)
+def test_tc_small_ragged(T, E, k, H, I, wq):
+    wl = BASE.replace(T=T, E=E, top_k=k, H=H, I=I, seed=T + E, wq=wq)
     inp = synth.make_inputs(wl)
     dev = to_device(wl, inp)
     out, ids = forward(wl, dev, "tc")
@@ -48,4 +49,16 @@ def test_tc_prefill_workload():
     ref = oracle.forward(wl, inp, rows=rows)
     assert np.array_equal(ids, ref["topk_ids"])
     err = rel_err(act_np(out)[rows], ref["out"])
+    assert err <= tol_for(wl), f"rel err {err:.3e}"
+
+
+def test_tc_sigmoid_grouped_fp8_with_shared_expert():
+    wl = BASE.replace(T=300, E=16, top_k=4, H=512, I=256, wq="fp8_b128", seed=31, score="sigmoid", routed_scale=2.5,
+                      n_group=4, topk_group=2, has_shared=True, I_shared=384, select_bias_sigma=0.01)
+    inp = synth.make_inputs(wl)
+    dev = to_device(wl, inp)
+    out, ids = forward(wl, dev, "tc")
+    ref = oracle.forward(wl, inp)
+    assert np.array_equal(ids.cpu().numpy(), ref["topk_ids"])
+    err = rel_err(act_np(out), ref["out"])
     assert err <= tol_for(wl), f"rel err {err:.3e}"
