@@ -310,21 +310,26 @@ def main():
     ffn_ms = fs.elapsed_time(fe) / args.steps
     pk, pk_kind = peaks()
     route = gb.ffn_route(cfg)
-    if route == "stream":
-        routed_bytes = algorithmic_weight_bytes(wl.replace(has_shared=False), active)
+    # the expert FFN's roofline: the slower of its algorithmic weight bytes over
+    # HBM bandwidth and its FLOPs over the bf16 tensor peak
+    routed_bytes = algorithmic_weight_bytes(wl.replace(has_shared=False), active)
+    flops = 6.0 * wl.P * wl.H * wl.I
+    t_hbm = routed_bytes / (pk["hbm_gbs"] * 1e9)
+    t_tensor = flops / (pk["bf16_tflops"] * 1e12)
+    kernel = {"stream": "moe_grouped_ffn, weight-streaming route (gate/up + down)",
+              "tc": "moe_grouped_ffn, tcgen05 route (row gather + gate/up GEMM with SwiGLU + down GEMM)",
+              "simt": "moe_grouped_ffn, CUDA-core route"}[route]
+    common = {"traffic": TRAFFIC.get((wl.name, route)), "kernel": kernel, "algorithmic_bytes": routed_bytes,
+              "algorithmic_flops": flops, "active_experts": active, "ms_per_launch": ffn_ms,
+              "roofline_ms": max(t_hbm, t_tensor) * 1e3}
+    if t_hbm >= t_tensor:
         achieved = routed_bytes / (ffn_ms / 1e3) / 1e9
         roofline = {"bound": "hbm", "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s",
-                    "frac": achieved / pk["hbm_gbs"], "traffic": TRAFFIC.get((wl.name, route)),
-                    "peak_kind": pk_kind, "kernel": "moe_grouped_ffn, weight-streaming route (gate/up + down)",
-                    "algorithmic_bytes": routed_bytes, "active_experts": active, "ms_per_launch": ffn_ms}
+                    "frac": achieved / pk["hbm_gbs"], "peak_kind": f"{pk_kind} HBM copy", **common}
     else:
-        flops = 6.0 * wl.P * wl.H * wl.I
         achieved = flops / (ffn_ms / 1e3) / 1e12
         roofline = {"bound": "tensor", "achieved": achieved, "peak": pk["bf16_tflops"], "unit": "TFLOP/s",
-                    "frac": achieved / pk["bf16_tflops"], "traffic": TRAFFIC.get((wl.name, route)),
-                    "peak_kind": f"{pk_kind} bf16 dense burst", "kernel": f"moe_grouped_ffn, {route} route "
-                    "(gather + gate/up GEMM with SwiGLU + down GEMM)", "algorithmic_flops": flops,
-                    "active_experts": active, "ms_per_launch": ffn_ms}
+                    "frac": achieved / pk["bf16_tflops"], "peak_kind": f"{pk_kind} bf16 dense burst", **common}
 
     # end to end through the public host-buffer entry point
     x_host = x.cpu().pin_memory()

@@ -14,7 +14,6 @@ using namespace gbmoe;
 namespace {
 
 constexpr size_t kAlign = 256;
-constexpr int kStreamRowsPerPass = 8;       // matches the streaming kernels' pass height
 constexpr size_t kSmemBudget = 227 * 1024;  // per-CTA shared memory on sm_103a
 
 size_t align_up(size_t v) { return (v + kAlign - 1) & ~(kAlign - 1); }
@@ -51,16 +50,13 @@ int check_cfg(const gbmoe_config* c) {
     return GBMOE_OK;
 }
 
-bool stream_fits(int H, int I, int act) {
-    return (size_t)kStreamRowsPerPass * H * act_bytes(act) <= kSmemBudget &&
-           (size_t)kStreamRowsPerPass * I * act_bytes(act) <= kSmemBudget;
-}
+bool stream_fits(int act_dtype, int H, int I) { return stream_smem_bytes(act_dtype, H, I) <= kSmemBudget; }
 
 // Kernel route for an FFN problem with n_rows rows over E experts.
 int pick_route(const gbmoe_config* c, int64_t n_rows, int E, int I) {
     int r = c->ffn_route;
     if (r != GBMOE_FFN_AUTO) return r;
-    if (n_rows <= 16 * (int64_t)E && stream_fits(c->H, I, c->act_dtype)) return GBMOE_FFN_STREAM;
+    if (n_rows <= 16 * (int64_t)E && stream_fits(c->act_dtype, c->H, I)) return GBMOE_FFN_STREAM;
     if (c->act_dtype == GBMOE_BF16) {
         FfnProblem probe{};
         probe.act_dtype = c->act_dtype;
@@ -140,7 +136,7 @@ int run_ffn(const gbmoe_config* c, FfnProblem& p, int route, cudaStream_t stream
     cudaError_t err;
     switch (route) {
         case GBMOE_FFN_STREAM:
-            if (!stream_fits(p.H, p.I, p.act_dtype)) return GBMOE_EUNSUPPORTED;
+            if (!stream_fits(p.act_dtype, p.H, p.I)) return GBMOE_EUNSUPPORTED;
             err = launch_ffn_stream(p, stream);
             break;
         case GBMOE_FFN_SIMT: err = launch_ffn_simt(p, stream); break;
@@ -307,7 +303,7 @@ int moe_forward(const gbmoe_config* cfg, const void* x, const void* w_router, co
     const int r_routed = pick_route(cfg, P, cfg->E, cfg->I);
     const int r_shared = cfg->has_shared ? pick_route(cfg, cfg->T, 1, cfg->I_shared) : GBMOE_FFN_SIMT;
     for (int r : {r_routed, r_shared}) {
-        if (r == GBMOE_FFN_STREAM && !stream_fits(cfg->H, r == r_routed ? cfg->I : cfg->I_shared, cfg->act_dtype))
+        if (r == GBMOE_FFN_STREAM && !stream_fits(cfg->act_dtype, cfg->H, r == r_routed ? cfg->I : cfg->I_shared))
             return GBMOE_EUNSUPPORTED;
     }
     if (cudaMemsetAsync(at<int32_t>(ws, L.err), 0, 4, st) != cudaSuccess) return GBMOE_ECUDA;

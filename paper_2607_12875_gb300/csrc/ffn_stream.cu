@@ -3,11 +3,14 @@
 // With ~2 rows per expert the layer is bound by reading each active expert's
 // weights once from HBM. Each CTA takes one active expert and a slice of
 // output columns; its warps stream weight rows with 16-byte non-allocating
-// loads (kUnroll chunks per row in flight per lane) and dot them against the
-// expert's activation rows, which sit in shared memory. Lane l takes the
-// 16-byte chunks l, l+32, ... of a row, so a warp reads 512 contiguous bytes
-// per row and step. Up to kNT rows are handled per weight pass; more rows
-// take further passes over the same weights.
+// loads (kUnroll chunks of each of its 4 rows in flight per lane: 8 KB per
+// warp) and dot them against the expert's activation rows, which sit in
+// shared memory. Lane l takes the 16-byte chunks l, l+32, ... of a row, so a
+// warp reads 512 contiguous bytes per row and step. The inner loop reloads
+// each activation chunk once and decodes the weights per activation row, so
+// the kernel stays within 128 registers and two CTAs (16 warps) share an SM.
+// Up to kNT rows are handled per weight pass; more rows take further passes
+// over the same weights.
 //   stage 1: h[r, i] = silu(x_r . Wgate[i]) * (x_r . Wup[i]), 2 columns per warp
 //   stage 2: y[r, n] = h_r . Wdown[n], 4 output columns per warp
 #include <type_traits>
@@ -22,6 +25,12 @@ namespace gbmoe {
 constexpr int kStreamWarps = 8;
 constexpr int kNT = 8;      // activation rows per weight pass
 constexpr int kUnroll = 4;  // chunks per row loaded before use
+
+// CTAs per SM the register budget is set for: two for bf16 weights (the
+// decode path); fp32 and quantised weights hold or decode more per element
+// and get the whole register file
+template <int WQ>
+constexpr int stream_min_blocks() { return WQ == GBMOE_BF16 ? 2 : 1; }
 
 // acc[q][r] += W_q . xs[r] for 4 weight rows q (byte pointers wrow, scale rows
 // srow) and NT activation rows r in shared memory (row stride K).
@@ -52,18 +61,18 @@ __device__ __forceinline__ void dot4(const uint8_t* const (&wrow)[4], const void
             for (int q = 0; q < 4; ++q) sc[q] = F::scale_at(srow[q], c * F::CE);
 #pragma unroll
             for (int sub = 0; sub < F::CE / 8; ++sub) {
-                float w[4][8];
-#pragma unroll
-                for (int q = 0; q < 4; ++q) F::decode8(raw[u][q], sub, sc[q], w[q]);
                 const int k0 = c * F::CE + 8 * sub;
 #pragma unroll
                 for (int r = 0; r < NT; ++r) {
                     float xv[8];
                     Vec8<TA>::load(xs + (size_t)r * K + k0, xv);
 #pragma unroll
-                    for (int q = 0; q < 4; ++q)
+                    for (int q = 0; q < 4; ++q) {
+                        float w[8];
+                        F::decode8(raw[u][q], sub, sc[q], w);
 #pragma unroll
-                        for (int i = 0; i < 8; ++i) acc[q][r] = fmaf(w[q][i], xv[i], acc[q][r]);
+                        for (int i = 0; i < 8; ++i) acc[q][r] = fmaf(w[i], xv[i], acc[q][r]);
+                    }
                 }
             }
         }
@@ -106,7 +115,7 @@ __device__ __forceinline__ void dispatch_nt(int nt, F&& f) {
 }
 
 template <typename TA, int WQ>
-__global__ void __launch_bounds__(kStreamWarps * 32)
+__global__ void __launch_bounds__(kStreamWarps * 32, stream_min_blocks<WQ>())
 stream_gateup_kernel(FfnProblem p) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     TA* xs = reinterpret_cast<TA*>(smem_raw);
@@ -152,7 +161,7 @@ stream_gateup_kernel(FfnProblem p) {
 }
 
 template <typename TA, int WQ>
-__global__ void __launch_bounds__(kStreamWarps * 32)
+__global__ void __launch_bounds__(kStreamWarps * 32, stream_min_blocks<WQ>())
 stream_down_kernel(FfnProblem p) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     TA* hs = reinterpret_cast<TA*>(smem_raw);
@@ -213,6 +222,12 @@ static cudaError_t launch_stream_t(const FfnProblem& p, cudaStream_t stream) {
     dim3 g2(max_active, p.H / (4 * kStreamWarps));
     stream_down_kernel<TA, WQ><<<g2, kStreamWarps * 32, smem2, stream>>>(p);
     return cudaGetLastError();
+}
+
+size_t stream_smem_bytes(int act_dtype, int H, int I) {
+    const size_t ab = act_dtype == GBMOE_F32 ? 4 : 2;
+    const size_t a = (size_t)kNT * H * ab, b = (size_t)kNT * I * ab;
+    return a > b ? a : b;
 }
 
 cudaError_t launch_ffn_stream(const FfnProblem& p, cudaStream_t stream) {

@@ -47,6 +47,7 @@ struct FfnProblem {
 
 size_t ffn_sched_ints(int E, int64_t n_rows);
 cudaError_t launch_ffn_stream(const FfnProblem& p, cudaStream_t stream);
+size_t stream_smem_bytes(int act_dtype, int H, int I);  // per CTA, streaming route
 cudaError_t launch_ffn_simt(const FfnProblem& p, cudaStream_t stream);
 cudaError_t launch_ffn_tc(const FfnProblem& p, cudaStream_t stream);
 bool ffn_tc_supported(const FfnProblem& p);
