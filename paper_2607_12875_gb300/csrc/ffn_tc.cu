@@ -470,30 +470,41 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
             int b0, b1;
             b_rows(p, wk, b0, b1);
             const int64_t brow = (half ? b1 : b0) + (r & 127);  // absolute row of the stacked B tensor
+            // scale of this row for 128-wide k group j: one per 128x128 block (fp8)
+            // or per row (int4), loaded four groups ahead so that no k-block waits
+            // on a global load before decoding
+            auto scale_of = [&](int j) -> float {
+                if (j >= kgroups) return 0.0f;
+                if (WQ == GBMOE_FP8_E4M3_B128) return static_cast<const float*>(scales)[(brow / 128) * kgroups + j];
+                return __bfloat162float(static_cast<const __nv_bfloat16*>(scales)[brow * kgroups + j]);
+            };
+            float sc0 = scale_of(0), sc1 = scale_of(1), sc2 = scale_of(2), sc3 = scale_of(3);
             for (int kb = 0; kb < nkb; ++kb) {
+                if (kb > 0 && (kb & 1) == 0) {  // next 128-wide group
+                    sc0 = sc1; sc1 = sc2; sc2 = sc3;
+                    sc3 = scale_of(kb / 2 + 3);
+                }
                 if (!mbar_wait(&full[stage], phase, abort_flag, p.err)) { ok = false; break; }
                 const uint8_t* raw = sR + stage * RAW;
                 uint8_t* dstB = sB + stage * B_BYTES;
                 if (WQ == GBMOE_FP8_E4M3_B128) {
-                    const float sc = static_cast<const float*>(scales)[(brow / 128) * kgroups + kb / 2];
 #pragma unroll
                     for (int c = 0; c < 4; ++c) {
                         const uint4 v = *reinterpret_cast<const uint4*>(raw + sw64_off(r, c));
                         uint4 o0, o1;
-                        decode_fp8_16(v, sc, o0, o1);
+                        decode_fp8_16(v, sc0, o0, o1);
                         *reinterpret_cast<uint4*>(dstB + sw128_off(r, 2 * c)) = o0;
                         *reinterpret_cast<uint4*>(dstB + sw128_off(r, 2 * c + 1)) = o1;
                     }
                 } else {
-                    const __nv_bfloat16 sb = static_cast<const __nv_bfloat16*>(scales)[brow * kgroups + kb / 2];
-                    const __nv_bfloat162 sc2 = __halves2bfloat162(sb, sb);
+                    const __nv_bfloat162 sc2v = __float2bfloat162_rn(sc0);  // exact: sc0 came from a bf16
 #pragma unroll
                     for (int c = 0; c < 2; ++c) {
                         const uint4 v = *reinterpret_cast<const uint4*>(raw + sw32_off(r, c));
                         const uint32_t ws[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
                         for (int i = 0; i < 4; ++i)
-                            *reinterpret_cast<uint4*>(dstB + sw128_off(r, 4 * c + i)) = decode_int4_8(ws[i], sc2);
+                            *reinterpret_cast<uint4*>(dstB + sw128_off(r, 4 * c + i)) = decode_int4_8(ws[i], sc2v);
                     }
                 }
                 // make the generic-proxy writes visible to the tensor core, then signal
