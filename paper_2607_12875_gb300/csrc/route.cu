@@ -6,7 +6,8 @@
 // butterfly of pairwise sums), so the expert choice is bit-identical to the
 // oracle's. A warp owns TB tokens x 8 experts; lane l holds the partial sums
 // of chunks l, l+32, ... for all of them, which is exactly the fixed order.
-// select_experts then runs one warp per token over the logits.
+// select_experts then runs one warp per token over the logits. Large batches
+// use a shared-memory-staged variant with the same order (below).
 #include "common.cuh"
 #include "kernels.h"
 
@@ -74,6 +75,118 @@ gate_logits_kernel(const TA* __restrict__ x, const TA* __restrict__ wg, const fl
         for (int b = 0; b < kGateExpertsPerWarp; ++b) {
             int t = t0 + a, e = e0 + b;
             if (lane == ((a * kGateExpertsPerWarp + b) & 31) && t < T && e < E) {
+                float l = acc[a][b];
+                if (bias) l = __fadd_rn(l, bias[e]);
+                logits[(size_t)t * E + e] = l;
+            }
+        }
+}
+
+// Large batches: the same fixed order, as a CUDA-core GEMM. A CTA owns 32
+// tokens x 16 experts; 256-element slabs of x and Wg go through a 3-stage
+// cp.async ring in shared memory, and warp w (of 8) accumulates tokens
+// 8*(w%4).. x experts 8*(w/4).. in registers. Lane l reads 8-element chunk l
+// of every slab, i.e. chunks l, l+32, ... in increasing order, elements in
+// increasing order inside a chunk, exactly as in the definition.
+constexpr int kGT = 32, kGE = 16, kSlab = 256, kGStages = 3;
+constexpr size_t kGateTiledSmem = (size_t)kGStages * (kGT + kGE) * kSlab * 2;
+
+__device__ __forceinline__ void cp_async16(void* dst, const void* src, bool valid) {
+    const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(dst));
+    const int n = valid ? 16 : 0;  // 0 bytes read: the 16 bytes are zero-filled
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(d), "l"(src), "r"(n) : "memory");
+}
+
+__global__ void __launch_bounds__(256, 1)
+gate_logits_tiled_kernel(const __nv_bfloat16* __restrict__ x, const __nv_bfloat16* __restrict__ wg,
+                         const float* __restrict__ bias, float* __restrict__ logits, int T, int H, int E) {
+    extern __shared__ __align__(16) uint8_t smem[];
+    uint8_t* sx = smem;                                          // [stage][kGT][kSlab] bf16
+    uint8_t* sw = smem + (size_t)kGStages * kGT * kSlab * 2;     // [stage][kGE][kSlab] bf16
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int t0 = blockIdx.x * kGT, e0 = blockIdx.y * kGE;
+    const int nslab = H / kSlab;
+
+    auto load_slab = [&](int j) {
+        const int st = j % kGStages;
+        // x: kGT rows x 32 chunks; Wg: kGE rows x 32 chunks; 16 bytes each
+        for (int i = threadIdx.x; i < (kGT + kGE) * 32; i += 256) {
+            const int row = i >> 5, c = i & 31;
+            if (row < kGT) {
+                const int t = t0 + row;
+                const bool ok = t < T;
+                cp_async16(sx + (((size_t)st * kGT + row) * kSlab + 8 * c) * 2,
+                           x + (size_t)(ok ? t : 0) * H + (size_t)j * kSlab + 8 * c, ok);
+            } else {
+                const int r = row - kGT, e = e0 + r;
+                const bool ok = e < E;
+                cp_async16(sw + (((size_t)st * kGE + r) * kSlab + 8 * c) * 2,
+                           wg + (size_t)(ok ? e : 0) * H + (size_t)j * kSlab + 8 * c, ok);
+            }
+        }
+    };
+
+    float acc[8][8];
+#pragma unroll
+    for (int a = 0; a < 8; ++a)
+#pragma unroll
+        for (int b = 0; b < 8; ++b) acc[a][b] = 0.0f;
+    const int tg = (warp & 3) * 8, eg = (warp >> 2) * 8;
+
+#pragma unroll
+    for (int j = 0; j < kGStages - 1; ++j) {
+        if (j < nslab) load_slab(j);
+        asm volatile("cp.async.commit_group;" ::: "memory");
+    }
+    for (int j = 0; j < nslab; ++j) {
+        asm volatile("cp.async.wait_group %0;" ::"n"(kGStages - 2) : "memory");
+        __syncthreads();
+        if (j + kGStages - 1 < nslab) load_slab(j + kGStages - 1);
+        asm volatile("cp.async.commit_group;" ::: "memory");
+        const int st = j % kGStages;
+        uint4 xr[8], wr[8];
+#pragma unroll
+        for (int a = 0; a < 8; ++a)
+            xr[a] = *reinterpret_cast<const uint4*>(sx + (((size_t)st * kGT + tg + a) * kSlab + 8 * lane) * 2);
+#pragma unroll
+        for (int b = 0; b < 8; ++b)
+            wr[b] = *reinterpret_cast<const uint4*>(sw + (((size_t)st * kGE + eg + b) * kSlab + 8 * lane) * 2);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            float xf[8], wf[8];
+#pragma unroll
+            for (int a = 0; a < 8; ++a) {
+                const uint32_t u = (&xr[a].x)[i >> 1];
+                xf[a] = (i & 1) ? bf16hi(u) : bf16lo(u);
+            }
+#pragma unroll
+            for (int b = 0; b < 8; ++b) {
+                const uint32_t u = (&wr[b].x)[i >> 1];
+                wf[b] = (i & 1) ? bf16hi(u) : bf16lo(u);
+            }
+#pragma unroll
+            for (int a = 0; a < 8; ++a)
+#pragma unroll
+                for (int b = 0; b < 8; ++b) acc[a][b] = __fmaf_rn(xf[a], wf[b], acc[a][b]);
+        }
+    }
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
+    // butterfly: s[p] <- s[p] + s[p ^ d], d = 16 .. 1
+#pragma unroll
+    for (int a = 0; a < 8; ++a)
+#pragma unroll
+        for (int b = 0; b < 8; ++b) {
+            float v = acc[a][b];
+#pragma unroll
+            for (int d = 16; d >= 1; d >>= 1) v = __fadd_rn(v, __shfl_xor_sync(0xffffffffu, v, d));
+            acc[a][b] = v;
+        }
+#pragma unroll
+    for (int a = 0; a < 8; ++a)
+#pragma unroll
+        for (int b = 0; b < 8; ++b) {
+            const int t = t0 + tg + a, e = e0 + eg + b;
+            if (lane == ((a * 8 + b) & 31) && t < T && e < E) {
                 float l = acc[a][b];
                 if (bias) l = __fadd_rn(l, bias[e]);
                 logits[(size_t)t * E + e] = l;
@@ -237,9 +350,12 @@ cudaError_t launch_route(const RouteParams& rp, const void* x, const void* wg, c
         auto xp = static_cast<const __nv_bfloat16*>(x);
         auto wp = static_cast<const __nv_bfloat16*>(wg);
         if (rp.T >= 1024) {
-            dim3 grid((rp.T + 7) / 8, ey);
-            gate_logits_kernel<__nv_bfloat16, 8><<<grid, block, 0, stream>>>(xp, wp, logit_bias, logits, rp.T,
-                                                                              rp.H, rp.E);
+            cudaError_t e = cudaFuncSetAttribute(gate_logits_tiled_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 (int)kGateTiledSmem);
+            if (e != cudaSuccess) return e;
+            dim3 grid((rp.T + kGT - 1) / kGT, (rp.E + kGE - 1) / kGE);
+            gate_logits_tiled_kernel<<<grid, 256, kGateTiledSmem, stream>>>(xp, wp, logit_bias, logits, rp.T, rp.H,
+                                                                            rp.E);
         } else {
             dim3 grid((rp.T + 1) / 2, ey);
             gate_logits_kernel<__nv_bfloat16, 2><<<grid, block, 0, stream>>>(xp, wp, logit_bias, logits, rp.T,
