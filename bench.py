@@ -126,8 +126,12 @@ class ClockSampler:
 
 # --------------------------------------------------------------- workload
 
-def load_workload(wid: int):
+def load_workload(wid: int, overrides=()):
+    """The workload and its inputs; overrides ("KEY=INT" strings) change its
+    shape, e.g. a reduced case for profiling."""
     wl = synth.WORKLOADS[wid]
+    if overrides:
+        wl = wl.replace(**{k: int(v) for k, v in (o.split("=", 1) for o in overrides)})
     inp = synth.make_inputs(wl)
     return wl, inp
 
@@ -197,6 +201,10 @@ def main():
     ap.add_argument("--route", default="auto", choices=["auto", "stream", "simt", "tc"])
     ap.add_argument("--ref-tokens", type=int, default=1, help="tokens per oracle step (reference arm)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--set", action="append", default=[], metavar="KEY=INT",
+                    help="override a workload field (reduced cases for profiling), e.g. --set T=2048 --set E=32")
+    ap.add_argument("--profile", type=int, default=0, metavar="N",
+                    help="run N untimed layer forwards and exit (for ncu captures); prints no bench line")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3
@@ -208,7 +216,7 @@ def main():
     if args.impl == "reference":
         if rank != 0:
             return
-        wl, inp = load_workload(args.workload)
+        wl, inp = load_workload(args.workload, args.set)
         print(json.dumps(run_reference(args, wl, inp, rank)))
         return
 
@@ -227,7 +235,7 @@ def main():
         if dist is not None:
             dist.barrier()
 
-    wl, inp = load_workload(args.workload)
+    wl, inp = load_workload(args.workload, args.set)
     dev = torch.device("cuda", local)
 
     def act(a):
@@ -257,6 +265,13 @@ def main():
 
     def step():
         gb.moe_forward(cfg, x, wr, lb, sb, experts, shared, out, ws)
+
+    if args.profile:
+        for _ in range(args.profile):
+            step()
+        torch.cuda.synchronize()
+        print(f"profile run: {wl.name} {args.set} route={gb.ffn_route(cfg)} status={gb.moe_device_status(ws)}")
+        return
 
     for _ in range(args.warmup):
         step()
