@@ -198,7 +198,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", type=int, default=2, help="synth.WORKLOADS id (2 = decode bf16)")
-    ap.add_argument("--route", default="auto", choices=["auto", "stream", "simt", "tc"])
+    ap.add_argument("--route", default="auto", choices=["auto", "stream", "simt", "tc", "tc_dequant"])
     ap.add_argument("--ref-tokens", type=int, default=1, help="tokens per oracle step (reference arm)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--set", action="append", default=[], metavar="KEY=INT",
@@ -333,6 +333,8 @@ def main():
     t_tensor = flops / (pk["bf16_tflops"] * 1e12)
     kernel = {"stream": "moe_grouped_ffn, weight-streaming route (gate/up + down)",
               "tc": "moe_grouped_ffn, tcgen05 route (row gather + gate/up GEMM with SwiGLU + down GEMM)",
+              "tc_dequant": "moe_grouped_ffn, tcgen05 decode-once route (3 weight-decode passes + row gather + "
+                            "gate/up GEMM with SwiGLU + down GEMM)",
               "simt": "moe_grouped_ffn, CUDA-core route"}[route]
     common = {"traffic": TRAFFIC.get((wl.name, route)), "kernel": kernel, "algorithmic_bytes": routed_bytes,
               "algorithmic_flops": flops, "active_experts": active, "ms_per_launch": ffn_ms,
@@ -369,8 +371,13 @@ def main():
 
     # kernels this library launched per step: gate logits + expert choice, 3 for the
     # permutation, per FFN problem a schedule kernel + 2 (+ a row gather for the routed experts on the
-    # tensor-core route), combine
-    per_step = 2 + 3 + (4 if route == "tc" else 3) + (3 if wl.has_shared else 0) + 1
+    # tensor-core routes, + 3 weight-decode passes on the decode-once route), combine
+    def ffn_launches(r, routed):
+        return 3 + (1 if routed and r in ("tc", "tc_dequant") else 0) + (3 if r == "tc_dequant" else 0)
+
+    per_step = 2 + 3 + ffn_launches(route, True) + 1
+    if wl.has_shared:
+        per_step += ffn_launches(gb.ffn_route(cfg, shared=True), False)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

@@ -64,12 +64,18 @@ enum { GBMOE_SOFTMAX = 0, GBMOE_SIGMOID = 1 };
 
 /* Which expert-FFN kernels run. AUTO streams weights when the average number
  * of rows per expert P/E is at most 16 and otherwise runs the grouped GEMM
- * (tensor cores for bf16 activations, CUDA cores for fp32). */
+ * (tensor cores for bf16 activations, CUDA cores for fp32). On the tensor
+ * cores, fp8/int4 weights are decoded inside the GEMM when P/E < 256; with
+ * more rows per expert (several M tiles reuse each weight tile) AUTO takes
+ * GBMOE_FFN_TC_DEQUANT: one pass decodes the active experts' weights to a
+ * bf16 copy in the workspace (the same bf16 values the in-GEMM decode makes),
+ * then the bf16 GEMM runs on it. */
 enum {
     GBMOE_FFN_AUTO = 0,
-    GBMOE_FFN_STREAM = 1, /* weight streaming: few rows per expert (decode)       */
-    GBMOE_FFN_SIMT = 2,   /* CUDA-core tiled GEMM (fp32 activations, any weights) */
-    GBMOE_FFN_TC = 3      /* tcgen05/TMEM/TMA grouped GEMM (bf16 activations)     */
+    GBMOE_FFN_STREAM = 1,     /* weight streaming: few rows per expert (decode)       */
+    GBMOE_FFN_SIMT = 2,       /* CUDA-core tiled GEMM (fp32 activations, any weights) */
+    GBMOE_FFN_TC = 3,         /* tcgen05/TMEM/TMA grouped GEMM (bf16 activations)     */
+    GBMOE_FFN_TC_DEQUANT = 4  /* as TC, quantised weights decoded once beforehand     */
 };
 
 typedef struct gbmoe_config {
@@ -114,7 +120,7 @@ int gbmoe_check_config(const gbmoe_config* cfg);
  * other calls need no more). 0 if the config is invalid. */
 size_t gbmoe_workspace_size(const gbmoe_config* cfg);
 
-/* The FFN route (GBMOE_FFN_STREAM, _SIMT or _TC) that moe_forward runs for
+/* The FFN route (GBMOE_FFN_STREAM, _SIMT, _TC or _TC_DEQUANT) that moe_forward runs for
  * cfg: for the routed experts (shared = 0) or the shared expert (shared = 1).
  * Negative status if the config is invalid. */
 int gbmoe_ffn_route(const gbmoe_config* cfg, int shared);

@@ -31,7 +31,7 @@ int check_cfg(const gbmoe_config* c) {
     if (c->w_dtype < GBMOE_F32 || c->w_dtype > GBMOE_INT4_G128) return GBMOE_EINVAL;
     if (c->has_shared != 0 && c->has_shared != 1) return GBMOE_EINVAL;
     if (c->has_shared && c->I_shared <= 0) return GBMOE_EINVAL;
-    if (c->ffn_route < GBMOE_FFN_AUTO || c->ffn_route > GBMOE_FFN_TC) return GBMOE_EINVAL;
+    if (c->ffn_route < GBMOE_FFN_AUTO || c->ffn_route > GBMOE_FFN_TC_DEQUANT) return GBMOE_EINVAL;
     if (!std::isfinite(c->routed_scale)) return GBMOE_EINVAL;
     if (c->score == GBMOE_SIGMOID) {
         if (c->n_group < 1 || c->E % c->n_group != 0) return GBMOE_EINVAL;
@@ -46,7 +46,8 @@ int check_cfg(const gbmoe_config* c) {
     if (c->score == GBMOE_SIGMOID && c->n_group > 32) return GBMOE_EUNSUPPORTED;
     if ((int64_t)c->T * c->top_k > (int64_t(1) << 30)) return GBMOE_EUNSUPPORTED;
     if (c->act_dtype == GBMOE_BF16 && c->w_dtype == GBMOE_F32) return GBMOE_EUNSUPPORTED;
-    if (c->ffn_route == GBMOE_FFN_TC && c->act_dtype != GBMOE_BF16) return GBMOE_EUNSUPPORTED;
+    if ((c->ffn_route == GBMOE_FFN_TC || c->ffn_route == GBMOE_FFN_TC_DEQUANT) && c->act_dtype != GBMOE_BF16)
+        return GBMOE_EUNSUPPORTED;
     return GBMOE_OK;
 }
 
@@ -64,13 +65,25 @@ int pick_route(const gbmoe_config* c, int64_t n_rows, int E, int I) {
         probe.H = c->H;
         probe.I = I;
         probe.E = E;
-        if (ffn_tc_supported(probe)) return GBMOE_FFN_TC;
+        if (ffn_tc_supported(probe)) {
+            const bool quantised = c->w_dtype == GBMOE_FP8_E4M3_B128 || c->w_dtype == GBMOE_INT4_G128;
+            return quantised && n_rows >= kDequantRowsPerExpert * E ? GBMOE_FFN_TC_DEQUANT : GBMOE_FFN_TC;
+        }
     }
     return GBMOE_FFN_SIMT;
 }
 
+// Bytes of the bf16 weight copy the TC_DEQUANT route decodes into (0 when
+// the route of that problem does not use one).
+size_t dequant_bytes(const gbmoe_config* c, int64_t n_rows, int E, int I) {
+    const bool quantised = c->w_dtype == GBMOE_FP8_E4M3_B128 || c->w_dtype == GBMOE_INT4_G128;
+    if (!quantised || pick_route(c, n_rows, E, I) != GBMOE_FFN_TC_DEQUANT) return 0;
+    return (size_t)3 * E * c->H * I * 2;
+}
+
 struct Layout {
-    size_t err, logits, ids, w, counts, offsets, sorted, pos, perm, sched, h, xs, y, ysh, xin, xout, total;
+    size_t err, logits, ids, w, counts, offsets, sorted, pos, perm, sched, h, xs, y, ysh, xin, xout, wdq, wdq_sh,
+        total;
 };
 
 Layout layout(const gbmoe_config* c) {
@@ -97,6 +110,8 @@ Layout layout(const gbmoe_config* c) {
     L.ysh = take(c->has_shared ? (size_t)T * H * ab : 0);
     L.xin = take((size_t)T * H * ab);
     L.xout = take((size_t)T * H * ab);
+    L.wdq = take(dequant_bytes(c, P, (int)E, c->I));
+    L.wdq_sh = take(c->has_shared ? dequant_bytes(c, T, 1, c->I_shared) : 0);
     L.total = o;
     return L;
 }
@@ -141,6 +156,7 @@ int run_ffn(const gbmoe_config* c, FfnProblem& p, int route, cudaStream_t stream
             break;
         case GBMOE_FFN_SIMT: err = launch_ffn_simt(p, stream); break;
         case GBMOE_FFN_TC:
+        case GBMOE_FFN_TC_DEQUANT:
             if (!ffn_tc_supported(p)) return GBMOE_EUNSUPPORTED;
             err = launch_ffn_tc(p, stream);
             break;
@@ -162,6 +178,7 @@ FfnProblem routed_problem(const gbmoe_config* c, const void* x, const int32_t* c
     p.y = y;
     p.h = at<char>(ws, L.h); p.x_sorted = at<char>(ws, L.xs); p.sched = at<int32_t>(ws, L.sched);
     p.err = at<int32_t>(ws, L.err);
+    p.w_dq = dequant_bytes(c, p.n_rows, p.E, p.I) ? at<char>(ws, L.wdq) : nullptr;
     return p;
 }
 
@@ -176,6 +193,7 @@ FfnProblem shared_problem(const gbmoe_config* c, const void* x, const gbmoe_expe
     p.y = y;
     p.h = at<char>(ws, L.h); p.x_sorted = at<char>(ws, L.xs); p.sched = at<int32_t>(ws, L.sched);
     p.err = at<int32_t>(ws, L.err);
+    p.w_dq = dequant_bytes(c, p.n_rows, p.E, p.I) ? at<char>(ws, L.wdq_sh) : nullptr;
     return p;
 }
 

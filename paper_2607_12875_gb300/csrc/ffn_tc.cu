@@ -538,6 +538,47 @@ gather_rows_kernel(const uint4* __restrict__ x, const int32_t* __restrict__ sort
     }
 }
 
+// ------------------------------------- one-pass decode of quantised weights
+
+// Active experts' quantised [N, K] matrices -> bf16 [E, N, K]. Each thread
+// decodes 16-byte raw chunks (16 fp8 or 32 int4 weights) with the same
+// functions and scale handling as the GEMM's converter warps, so the copy
+// holds exactly the bf16 operands the in-GEMM decode would produce.
+template <int WQ>
+__global__ void __launch_bounds__(256)
+dequant_weights_kernel(const uint8_t* __restrict__ w, const void* __restrict__ s, int N, int K,
+                       const int32_t* __restrict__ sched, __nv_bfloat16* __restrict__ out) {
+    const int slot = blockIdx.y;
+    if (slot >= sched[0]) return;
+    const int64_t e = sched[kSchedHeader + slot];
+    constexpr bool kFp8 = WQ == GBMOE_FP8_E4M3_B128;
+    constexpr int EPC = kFp8 ? 16 : 32;  // weights per 16-byte raw chunk
+    const int cpr = K / EPC;
+    const int64_t nchunks = (int64_t)N * cpr;
+    const uint8_t* src = w + e * N * (int64_t)(kFp8 ? K : K / 2);
+    __nv_bfloat16* dst_e = out + e * N * (int64_t)K;
+    for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < nchunks; c += (int64_t)gridDim.x * blockDim.x) {
+        const int n = (int)(c / cpr);
+        const int k0 = (int)(c - (int64_t)n * cpr) * EPC;
+        const uint4 raw = ld_stream16(src + c * 16);
+        uint4* dst = reinterpret_cast<uint4*>(dst_e + (int64_t)n * K + k0);
+        if constexpr (kFp8) {
+            const float sc = static_cast<const float*>(s)[(e * (N / 128) + n / 128) * (K / 128) + k0 / 128];
+            uint4 o0, o1;
+            decode_fp8_16(raw, sc, o0, o1);
+            dst[0] = o0;
+            dst[1] = o1;
+        } else {
+            const float sc = __bfloat162float(static_cast<const __nv_bfloat16*>(s)[(e * N + n) * (K / 128) + k0 / 128]);
+            const __nv_bfloat162 sc2 = __float2bfloat162_rn(sc);
+            dst[0] = decode_int4_8(raw.x, sc2);
+            dst[1] = decode_int4_8(raw.y, sc2);
+            dst[2] = decode_int4_8(raw.z, sc2);
+            dst[3] = decode_int4_8(raw.w, sc2);
+        }
+    }
+}
+
 // ------------------------------------------------------------------- host
 
 using EncodeTiled = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
@@ -625,11 +666,43 @@ bool ffn_tc_supported(const FfnProblem& p) {
     return p.act_dtype == GBMOE_BF16 && wq_ok && p.H % 256 == 0 && p.I % 128 == 0 && tc::encode_fn() != nullptr;
 }
 
-cudaError_t launch_ffn_tc(const FfnProblem& p, cudaStream_t stream) {
+// Decodes gate, up and down of the active experts into the bf16 copy w_dq
+// and returns the problem with its weights pointing there.
+static cudaError_t dequant_all(const FfnProblem& p, FfnProblem& q, cudaStream_t stream) {
     using namespace tc;
-    if (p.n_rows == 0) return cudaSuccess;
-    cudaError_t err = launch_ffn_schedule(p.counts, p.E, p.n_rows, BM, p.sched, stream);
+    q = p;
+    __nv_bfloat16* dq = static_cast<__nv_bfloat16*>(p.w_dq);
+    const int64_t gu = (int64_t)p.E * p.I * p.H;
+    struct Part { const void* w; const void* s; int N, K; __nv_bfloat16* out; };
+    const Part parts[3] = {{p.w_gate, p.s_gate, p.I, p.H, dq}, {p.w_up, p.s_up, p.I, p.H, dq + gu},
+                           {p.w_down, p.s_down, p.H, p.I, dq + 2 * gu}};
+    for (const Part& pt : parts) {
+        const int64_t nchunks = (int64_t)pt.N * pt.K / (p.w_dtype == GBMOE_FP8_E4M3_B128 ? 16 : 32);
+        const dim3 grid((unsigned)min64((nchunks + 1023) / 1024, 4096), (unsigned)p.E);
+        if (p.w_dtype == GBMOE_FP8_E4M3_B128)
+            dequant_weights_kernel<GBMOE_FP8_E4M3_B128><<<grid, 256, 0, stream>>>(
+                static_cast<const uint8_t*>(pt.w), pt.s, pt.N, pt.K, p.sched, pt.out);
+        else
+            dequant_weights_kernel<GBMOE_INT4_G128><<<grid, 256, 0, stream>>>(
+                static_cast<const uint8_t*>(pt.w), pt.s, pt.N, pt.K, p.sched, pt.out);
+        const cudaError_t err = cudaGetLastError();
+        if (err != cudaSuccess) return err;
+    }
+    q.w_dtype = GBMOE_BF16;
+    q.w_gate = dq; q.w_up = dq + gu; q.w_down = dq + 2 * gu;
+    q.s_gate = q.s_up = q.s_down = nullptr;
+    q.w_dq = nullptr;
+    return cudaSuccess;
+}
+
+cudaError_t launch_ffn_tc(const FfnProblem& pin, cudaStream_t stream) {
+    using namespace tc;
+    if (pin.n_rows == 0) return cudaSuccess;
+    cudaError_t err = launch_ffn_schedule(pin.counts, pin.E, pin.n_rows, BM, pin.sched, stream);
     if (err != cudaSuccess) return err;
+    FfnProblem p = pin;
+    if (pin.w_dq && (pin.w_dtype == GBMOE_FP8_E4M3_B128 || pin.w_dtype == GBMOE_INT4_G128))
+        if ((err = dequant_all(pin, p, stream)) != cudaSuccess) return err;
     // A operand of the gate/up GEMM: x rows in sorted order (a gathered copy),
     // or x itself when rows are already in order (no sorted_pair: shared expert)
     const void* a_rows = p.x;

@@ -41,11 +41,14 @@ struct FfnProblem {
     // scratch carved by the caller
     void* h;                    // [n_rows, I] act
     void* x_sorted;             // [n_rows, H] act (tensor-core route only)
+    void* w_dq;                 // bf16 [E, I, H] gate, [E, I, H] up, [E, H, I] down, or null:
+                                // quantised weights are then decoded once into it (TC_DEQUANT)
     int32_t* sched;             // schedule ints, ffn_sched_ints(E, n_rows)
     int32_t* err;               // device error word
 };
 
 size_t ffn_sched_ints(int E, int64_t n_rows);
+constexpr int64_t kDequantRowsPerExpert = 256;  // AUTO: TC_DEQUANT from this many rows per expert
 cudaError_t launch_ffn_stream(const FfnProblem& p, cudaStream_t stream);
 size_t stream_smem_bytes(int act_dtype, int H, int I);  // per CTA, streaming route
 cudaError_t launch_ffn_simt(const FfnProblem& p, cudaStream_t stream);

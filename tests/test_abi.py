@@ -68,6 +68,7 @@ def test_workload_configs_are_valid(lib, wid):
     (dict(act_dtype=2), gb.EINVAL),
     (dict(ffn_route=9), gb.EINVAL),
     (dict(ffn_route=gb.FFN_TC), gb.EUNSUPPORTED),  # fp32 activations have no tensor-core route
+    (dict(ffn_route=gb.FFN_TC_DEQUANT), gb.EUNSUPPORTED),
 ])
 def test_invalid_configs_are_rejected(lib, change, status):
     c = cfg_of(1, **change)
@@ -126,3 +127,14 @@ def test_entry_points_reject_bad_arguments_before_launching(lib):
         gb.moe_forward(c4, p, p, None, None, gb.weights(p, p, p), gb.weights(p, p, p), p, p, stream=0)  # no fp8 scales
     assert e.value.status == gb.EINVAL
     assert gb.status_string(gb.EDEVICE_TIMEOUT) == "device-side wait timed out"
+
+
+@pytest.mark.parametrize("wid", [4, 5])
+def test_dequant_route_workspace_holds_bf16_weight_copies(lib, wid):
+    """Forcing the decode-once route adds one bf16 copy of every expert's
+    gate, up and down matrices (and of the shared expert's) to the workspace."""
+    wl = synth.WORKLOADS[wid]
+    tc = gb.workspace_size(cfg_of(wid, ffn_route=gb.FFN_TC))
+    dq = gb.workspace_size(cfg_of(wid, ffn_route=gb.FFN_TC_DEQUANT))
+    copies = 3 * wl.E * wl.H * wl.I * 2 + (3 * wl.H * wl.I_shared * 2 if wl.has_shared else 0)
+    assert copies <= dq - tc <= copies + 2 * 256

@@ -16,7 +16,7 @@ pytestmark = pytest.mark.gpu
 # sampled-token counts for the big workloads (all tokens for the first two)
 SAMPLE = {3: (48, 16), 4: (20, 6), 5: (40, 12)}
 ROUTES = {1: ["simt", "stream", "auto"], 2: ["stream", "simt", "auto"], 3: ["simt", "auto"],
-          4: ["simt", "auto"], 5: ["simt", "auto"]}
+          4: ["simt", "auto", "tc_dequant"], 5: ["simt", "auto", "tc"]}
 
 _cache = {}
 

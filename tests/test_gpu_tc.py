@@ -1,5 +1,6 @@
-"""GPU parity of the tensor-core (tcgen05) grouped-GEMM route against the
-oracle: small ragged problems first, then the prefill-shaped workload."""
+"""GPU parity of the tensor-core (tcgen05) grouped-GEMM routes against the
+oracle: small ragged problems first, then the prefill-shaped workload; the
+decode-once route (TC_DEQUANT) against the in-GEMM decode."""
 import numpy as np
 import pytest
 import torch
@@ -15,6 +16,7 @@ BASE = synth.WORKLOADS[1].replace(act="bf16", wq="bf16")
 
 
 def forward(wl, dev, route):
+    """moe_forward of wl on the given FFN route; returns (out, topk_ids)."""
     cfg = config(wl, route)
     ws = workspace(cfg)
     out = torch.empty((wl.T, wl.H), dtype=torch.bfloat16, device="cuda")
@@ -62,3 +64,44 @@ def test_tc_sigmoid_grouped_fp8_with_shared_expert():
     assert np.array_equal(ids.cpu().numpy(), ref["topk_ids"])
     err = rel_err(act_np(out), ref["out"])
     assert err <= tol_for(wl), f"rel err {err:.3e}"
+
+
+@pytest.mark.parametrize("wq", ["fp8_b128", "int4_g128"])
+@pytest.mark.parametrize("T,E,k,H,I", [(200, 4, 2, 512, 256), (333, 16, 3, 768, 128)])
+def test_dequant_route_equals_in_gemm_decode(T, E, k, H, I, wq):
+    """Decoding the weights once into a bf16 copy gives the GEMM the same bf16
+    operands as decoding them inside it, so the outputs are bit-identical."""
+    wl = BASE.replace(T=T, E=E, top_k=k, H=H, I=I, seed=T + 2 * E, wq=wq)
+    inp = synth.make_inputs(wl)
+    dev = to_device(wl, inp)
+    out_tc, ids_tc = forward(wl, dev, "tc")
+    out_dq, ids_dq = forward(wl, dev, "tc_dequant")
+    assert torch.equal(ids_tc, ids_dq)
+    assert torch.equal(out_tc.view(torch.int16), out_dq.view(torch.int16))
+    ref = oracle.forward(wl, inp)
+    err = rel_err(act_np(out_dq), ref["out"])
+    assert err <= tol_for(wl), f"rel err {err:.3e}"
+
+
+def test_dequant_route_with_shared_expert_and_inactive_experts():
+    """Only active experts are decoded; the shared expert has its own copy."""
+    wl = BASE.replace(T=60, E=64, top_k=2, H=512, I=256, wq="int4_g128", seed=57, has_shared=True, I_shared=384,
+                      zipf=True)
+    inp = synth.make_inputs(wl)
+    dev = to_device(wl, inp)
+    out, ids = forward(wl, dev, "tc_dequant")
+    ref = oracle.forward(wl, inp)
+    assert (ref["counts"] == 0).any()
+    assert np.array_equal(ids.cpu().numpy(), ref["topk_ids"])
+    err = rel_err(act_np(out), ref["out"])
+    assert err <= tol_for(wl), f"rel err {err:.3e}"
+
+
+def test_auto_route_choice():
+    """AUTO: streaming for decode, in-GEMM decode for few rows per expert,
+    decode-once for many."""
+    assert gb.ffn_route(config(synth.WORKLOADS[2])) == "stream"
+    assert gb.ffn_route(config(synth.WORKLOADS[3])) == "tc"
+    assert gb.ffn_route(config(synth.WORKLOADS[4])) == "tc"
+    assert gb.ffn_route(config(synth.WORKLOADS[4]), shared=True) == "tc_dequant"
+    assert gb.ffn_route(config(synth.WORKLOADS[5])) == "tc_dequant"
