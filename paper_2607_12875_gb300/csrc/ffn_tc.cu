@@ -45,6 +45,7 @@ constexpr int B_BYTES = BN * BK * 2;
 constexpr int TMEM_COLS = 512;
 constexpr int CONVERT_WARPS = 8;  // one thread per B row (BN = 256)
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;
+constexpr int kFp8PrefetchAhead = 4;  // k-blocks the fp8 producer prefetches into L2 ahead of its loads
 
 // Per weight format: bytes of the raw B tile TMA brings in (0 = B is loaded
 // as bf16 directly), pipeline depth, threads.
@@ -68,7 +69,11 @@ struct Layout {
     static constexpr int STAGES = Fmt<WQ>::STAGES;
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES + Fmt<WQ>::RAW_BYTES;
     static constexpr int NUM_BARS = 3 * STAGES + 4 + 1;
-    static constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + NUM_BARS * 8 + 16;
+    static constexpr int BASE_BYTES = 1024 + STAGES * STAGE_BYTES + NUM_BARS * 8 + 16;
+    // output staging for TMA stores: 4 epilogue warps x 2 buffers x (32 rows x 64 bytes),
+    // when it fits next to the ring (otherwise the epilogue stores from registers)
+    static constexpr int EPI_BYTES = BASE_BYTES + 4 * 2 * 2048 <= 232448 ? 4 * 2 * 2048 : 0;
+    static constexpr int SMEM_BYTES = BASE_BYTES + EPI_BYTES;
     static_assert(SMEM_BYTES <= 232448, "shared memory per CTA");
 };
 
@@ -150,6 +155,26 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, i
         : "memory");
 }
 
+// Shared -> global TMA store of one box, tracked by the issuing thread's bulk groups
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void* src, int x, int y) {
+    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
+                     reinterpret_cast<uint64_t>(map)),
+                 "r"(x), "r"(y), "r"(smem_u32(src))
+                 : "memory");
+    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+// at most N of this thread's bulk stores still reading shared memory
+template <int N>
+__device__ __forceinline__ void bulk_wait_read() { asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory"); }
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
+// L2 prefetch of one box of a tensor map (no shared-memory destination)
+__device__ __forceinline__ void tma_prefetch_2d(const CUtensorMap* map, int x, int y) {
+    asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(reinterpret_cast<uint64_t>(map)),
+                 "r"(x), "r"(y)
+                 : "memory");
+}
+
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
@@ -201,6 +226,20 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 #pragma unroll
     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// 32 fp32 -> 32 bf16 into row `lane` of a 32-row x 64-byte staging buffer in
+// the 64-byte-swizzled layout TMA reads for a {32 columns, 32 rows} box
+__device__ __forceinline__ void stage_bf16x32(uint8_t* buf, int lane, const float (&v)[32]) {
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        uint4 u;
+        u.x = pack_bf16x2(v[8 * q + 0], v[8 * q + 1]);
+        u.y = pack_bf16x2(v[8 * q + 2], v[8 * q + 3]);
+        u.z = pack_bf16x2(v[8 * q + 4], v[8 * q + 5]);
+        u.w = pack_bf16x2(v[8 * q + 6], v[8 * q + 7]);
+        *reinterpret_cast<uint4*>(buf + lane * 64 + ((q ^ ((lane >> 1) & 3)) << 4)) = u;
+    }
 }
 
 __device__ __forceinline__ void store_bf16x32(__nv_bfloat16* dst, const float (&v)[32]) {
@@ -297,7 +336,7 @@ __device__ __forceinline__ void b_rows(const Params& p, const Work& wk, int& b0,
 template <int WQ>
 __global__ void __launch_bounds__(Fmt<WQ>::THREADS, 1)
 tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b0,
-               const __grid_constant__ CUtensorMap tm_b1, const Params p) {
+               const __grid_constant__ CUtensorMap tm_b1, const __grid_constant__ CUtensorMap tm_out, const Params p) {
     using L = Layout<WQ>;
     constexpr int STAGES = L::STAGES;
     constexpr int RAW = Fmt<WQ>::RAW_BYTES;
@@ -306,7 +345,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
     uint8_t* sA = smem;
     uint8_t* sB = smem + STAGES * A_BYTES;
     uint8_t* sR = smem + STAGES * (A_BYTES + B_BYTES);  // raw quantised B tiles
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * L::STAGE_BYTES);
+    uint8_t* sE = smem + STAGES * L::STAGE_BYTES;  // output staging (L::EPI_BYTES)
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sE + L::EPI_BYTES);
     uint64_t* full = bars;                 // TMA landed (A + B or A + raw B)
     uint64_t* empty = bars + STAGES;       // MMAs reading the slot finished
     uint64_t* conv = bars + 2 * STAGES;    // bf16 B written by the converters
@@ -356,6 +396,14 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
             int b0, b1;
             b_rows(p, wk, b0, b1);
             for (int kb = 0; kb < nkb; ++kb) {
+                if (WQ == GBMOE_FP8_E4M3_B128 && kb + kFp8PrefetchAhead < nkb) {
+                    // fp8 tiles wait on the decode as well as on the load: bring the
+                    // k-block a few stages ahead into L2 so its TMA load returns sooner
+                    const int xp = (kb + kFp8PrefetchAhead) * BK;
+                    tma_prefetch_2d(&tm_a, xp, (int)wk.row0);
+                    tma_prefetch_2d(&tm_b0, xp, b0);
+                    tma_prefetch_2d(&tm_b1, xp, b1);
+                }
                 if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, p.err)) { ok = false; break; }
                 inflight &= ~(1u << stage);
                 mbar_expect_tx(&full[stage], A_BYTES + (RAW ? RAW : B_BYTES));
@@ -423,6 +471,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
         // -------------------------------------------------------- epilogue
         const int q = warp & 3;       // TMEM lane quarter of this warp
         const int r = q * 32 + lane;  // tile row of this thread
+        uint8_t* stage_buf = sE + q * 4096;  // two 2 KB buffers of this warp
+        int sbuf = 0;
         int acc = 0;
         uint32_t acc_phase = 0;
         for (int w = blockIdx.x; w < total; w += gridDim.x) {
@@ -431,31 +481,41 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
             tc_fence_after();
             const uint32_t t_row = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
             const bool valid = r < wk.rows;
-            __nv_bfloat16* dst = p.out + (wk.row0 + r) * (int64_t)p.out_cols;
-            if (p.swiglu) {
-                dst += wk.nt * (BN / 2);
+            // all 32 rows of this warp belong to the tile: one TMA store per 32 columns;
+            // otherwise plain stores of the valid rows only (the rows past the tile's end
+            // belong to the next expert and are written by another tile)
+            const bool via_tma = L::EPI_BYTES > 0 && q * 32 + 32 <= wk.rows;
+            const int col0 = p.swiglu ? wk.nt * (BN / 2) : wk.nt * BN;
+            __nv_bfloat16* dst = p.out + (wk.row0 + r) * (int64_t)p.out_cols + col0;
+            const int ncols = p.swiglu ? BN / 2 : BN;
 #pragma unroll 1
-                for (int c = 0; c < BN / 2; c += 32) {
-                    float g[32], u[32];
-                    tmem_ld32(t_row + c, g);
+            for (int c = 0; c < ncols; c += 32) {
+                float v[32];
+                tmem_ld32(t_row + c, v);
+                if (p.swiglu) {
+                    float u[32];
                     tmem_ld32(t_row + BN / 2 + c, u);
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) g[i] = silu_mul(g[i], u[i]);
-                    if (valid) store_bf16x32(dst + c, g);
+                    for (int i = 0; i < 32; ++i) v[i] = silu_mul(v[i], u[i]);
                 }
-            } else {
-                dst += wk.nt * BN;
-#pragma unroll 1
-                for (int c = 0; c < BN; c += 32) {
-                    float v[32];
-                    tmem_ld32(t_row + c, v);
-                    if (valid) store_bf16x32(dst + c, v);
+                if (via_tma) {
+                    uint8_t* buf = stage_buf + sbuf * 2048;
+                    if (lane == 0) bulk_wait_read<1>();  // the store that last read buf is done reading
+                    __syncwarp();
+                    stage_bf16x32(buf, lane, v);
+                    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                    __syncwarp();
+                    if (lane == 0) tma_store_2d(&tm_out, buf, col0 + c, (int)(wk.row0 + q * 32));
+                    sbuf ^= 1;
+                } else if (valid) {
+                    store_bf16x32(dst + c, v);
                 }
             }
             tc_fence_before();
             mbar_arrive(&tempty[acc]);
             if (++acc == 2) { acc = 0; acc_phase ^= 1; }
         }
+        if (lane == 0) bulk_wait_all();  // stores complete before the CTA exits
     } else if (RAW && warp >= 6) {
         // ------------------------------------------- weight decode (B rows)
         const int r = threadIdx.x - 6 * 32;  // B row 0..255 of the tile
@@ -601,14 +661,14 @@ static EncodeTiled encode_fn() {
 }
 
 // 2-D row-major matrix [rows, row_bytes / elem] in boxes of box_x elements x
-// 128 rows with the given swizzle
+// box_rows rows with the given swizzle
 static bool make_map(CUtensorMap* m, const void* base, int64_t rows, int64_t row_bytes, CUtensorMapDataType dt,
-                     int elem_bytes, int box_x, CUtensorMapSwizzle sw) {
+                     int elem_bytes, int box_x, CUtensorMapSwizzle sw, int box_rows = 128) {
     EncodeTiled fn = encode_fn();
     if (!fn) return false;
     cuuint64_t dims[2] = {(cuuint64_t)(row_bytes / elem_bytes), (cuuint64_t)rows};
     cuuint64_t strides[1] = {(cuuint64_t)row_bytes};
-    cuuint32_t box[2] = {(cuuint32_t)box_x, 128};
+    cuuint32_t box[2] = {(cuuint32_t)box_x, (cuuint32_t)box_rows};
     cuuint32_t estr[2] = {1, 1};
     return fn(m, dt, 2, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, sw,
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
@@ -616,6 +676,11 @@ static bool make_map(CUtensorMap* m, const void* base, int64_t rows, int64_t row
 
 static bool map_bf16(CUtensorMap* m, const void* base, int64_t rows, int64_t cols) {
     return make_map(m, base, rows, cols * 2, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, BK, CU_TENSOR_MAP_SWIZZLE_128B);
+}
+
+// GEMM output [rows, cols] bf16 in {32 columns, 32 rows} boxes, 64-byte swizzle (epilogue TMA stores)
+static bool map_out(CUtensorMap* m, const void* base, int64_t rows, int64_t cols) {
+    return make_map(m, base, rows, cols * 2, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, 32, CU_TENSOR_MAP_SWIZZLE_64B, 32);
 }
 
 // B operand [rows, K] in the weight format WQ
@@ -639,22 +704,23 @@ static int num_sms() {
 
 template <int WQ>
 static cudaError_t launch_gemm_t(const CUtensorMap& a, const CUtensorMap& b0, const CUtensorMap& b1,
-                                 const Params& prm, int64_t max_work, cudaStream_t stream) {
+                                 const CUtensorMap& out, const Params& prm, int64_t max_work, cudaStream_t stream) {
     cudaError_t e = cudaFuncSetAttribute(tc_gemm_kernel<WQ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          Layout<WQ>::SMEM_BYTES);
     if (e != cudaSuccess) return e;
     const int grid = (int)min64(num_sms(), max_work);
     if (grid <= 0) return cudaSuccess;
-    tc_gemm_kernel<WQ><<<grid, Fmt<WQ>::THREADS, Layout<WQ>::SMEM_BYTES, stream>>>(a, b0, b1, prm);
+    tc_gemm_kernel<WQ><<<grid, Fmt<WQ>::THREADS, Layout<WQ>::SMEM_BYTES, stream>>>(a, b0, b1, out, prm);
     return cudaGetLastError();
 }
 
 static cudaError_t launch_gemm(int wq, const CUtensorMap& a, const CUtensorMap& b0, const CUtensorMap& b1,
-                               const Params& prm, int64_t max_work, cudaStream_t stream) {
+                               const CUtensorMap& out, const Params& prm, int64_t max_work, cudaStream_t stream) {
     switch (wq) {
-        case GBMOE_BF16: return launch_gemm_t<GBMOE_BF16>(a, b0, b1, prm, max_work, stream);
-        case GBMOE_FP8_E4M3_B128: return launch_gemm_t<GBMOE_FP8_E4M3_B128>(a, b0, b1, prm, max_work, stream);
-        case GBMOE_INT4_G128: return launch_gemm_t<GBMOE_INT4_G128>(a, b0, b1, prm, max_work, stream);
+        case GBMOE_BF16: return launch_gemm_t<GBMOE_BF16>(a, b0, b1, out, prm, max_work, stream);
+        case GBMOE_FP8_E4M3_B128:
+            return launch_gemm_t<GBMOE_FP8_E4M3_B128>(a, b0, b1, out, prm, max_work, stream);
+        case GBMOE_INT4_G128: return launch_gemm_t<GBMOE_INT4_G128>(a, b0, b1, out, prm, max_work, stream);
         default: return cudaErrorInvalidValue;
     }
 }
@@ -717,10 +783,11 @@ cudaError_t launch_ffn_tc(const FfnProblem& pin, cudaStream_t stream) {
     }
 
     const int64_t max_m = sched_max_tiles(p.E, p.n_rows, BM);
-    CUtensorMap ma, mg, mu, mh, md;
+    CUtensorMap ma, mg, mu, mh, md, oh, oy;
     if (!map_bf16(&ma, a_rows, p.n_rows, p.H) || !map_weights(&mg, p.w_dtype, p.w_gate, (int64_t)p.E * p.I, p.H) ||
         !map_weights(&mu, p.w_dtype, p.w_up, (int64_t)p.E * p.I, p.H) || !map_bf16(&mh, p.h, p.n_rows, p.I) ||
-        !map_weights(&md, p.w_dtype, p.w_down, (int64_t)p.E * p.H, p.I))
+        !map_weights(&md, p.w_dtype, p.w_down, (int64_t)p.E * p.H, p.I) || !map_out(&oh, p.h, p.n_rows, p.I) ||
+        !map_out(&oy, p.y, p.n_rows, p.H))
         return cudaErrorInvalidValue;
 
     Params g{};
@@ -728,13 +795,13 @@ cudaError_t launch_ffn_tc(const FfnProblem& pin, cudaStream_t stream) {
     g.counts = p.counts; g.offsets = p.offsets; g.sched = p.sched; g.E = p.E; g.n_rows = p.n_rows;
     g.out = static_cast<__nv_bfloat16*>(p.h); g.err = p.err;
     g.scale0 = p.s_gate; g.scale1 = p.s_up;
-    if ((err = launch_gemm(p.w_dtype, ma, mg, mu, g, max_m * g.n_tiles, stream)) != cudaSuccess) return err;
+    if ((err = launch_gemm(p.w_dtype, ma, mg, mu, oh, g, max_m * g.n_tiles, stream)) != cudaSuccess) return err;
 
     Params d = g;
     d.K = p.I; d.n_tiles = p.H / BN; d.out_cols = p.H; d.b_rows_per_expert = p.H; d.swiglu = 0;
     d.out = static_cast<__nv_bfloat16*>(p.y);
     d.scale0 = p.s_down; d.scale1 = p.s_down;
-    return launch_gemm(p.w_dtype, mh, md, md, d, max_m * d.n_tiles, stream);
+    return launch_gemm(p.w_dtype, mh, md, md, oy, d, max_m * d.n_tiles, stream);
 }
 
 }  // namespace gbmoe
