@@ -600,10 +600,14 @@ gather_rows_kernel(const uint4* __restrict__ x, const int32_t* __restrict__ sort
 
 // ------------------------------------- one-pass decode of quantised weights
 
-// Active experts' quantised [N, K] matrices -> bf16 [E, N, K]. Each thread
-// decodes 16-byte raw chunks (16 fp8 or 32 int4 weights) with the same
-// functions and scale handling as the GEMM's converter warps, so the copy
-// holds exactly the bf16 operands the in-GEMM decode would produce.
+// Active experts' quantised [N, K] matrices -> bf16 [E, N, K]. A thread
+// decodes 8 consecutive weights at a time (8 fp8 bytes or one 32-bit word of
+// int4) into one 16-byte bf16 chunk, so a warp reads 256 or 128 contiguous
+// bytes and writes 512; each thread first loads kDqUnroll such pieces. The
+// decode functions and scale handling are the GEMM converter warps', so the
+// copy holds exactly the bf16 operands the in-GEMM decode would produce.
+constexpr int kDqUnroll = 4;
+
 template <int WQ>
 __global__ void __launch_bounds__(256)
 dequant_weights_kernel(const uint8_t* __restrict__ w, const void* __restrict__ s, int N, int K,
@@ -612,29 +616,41 @@ dequant_weights_kernel(const uint8_t* __restrict__ w, const void* __restrict__ s
     if (slot >= sched[0]) return;
     const int64_t e = sched[kSchedHeader + slot];
     constexpr bool kFp8 = WQ == GBMOE_FP8_E4M3_B128;
-    constexpr int EPC = kFp8 ? 16 : 32;  // weights per 16-byte raw chunk
-    const int cpr = K / EPC;
-    const int64_t nchunks = (int64_t)N * cpr;
+    const int64_t npieces = (int64_t)N * K / 8;  // 8 weights each
     const uint8_t* src = w + e * N * (int64_t)(kFp8 ? K : K / 2);
-    __nv_bfloat16* dst_e = out + e * N * (int64_t)K;
-    for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < nchunks; c += (int64_t)gridDim.x * blockDim.x) {
-        const int n = (int)(c / cpr);
-        const int k0 = (int)(c - (int64_t)n * cpr) * EPC;
-        const uint4 raw = ld_stream16(src + c * 16);
-        uint4* dst = reinterpret_cast<uint4*>(dst_e + (int64_t)n * K + k0);
-        if constexpr (kFp8) {
-            const float sc = static_cast<const float*>(s)[(e * (N / 128) + n / 128) * (K / 128) + k0 / 128];
-            uint4 o0, o1;
-            decode_fp8_16(raw, sc, o0, o1);
-            dst[0] = o0;
-            dst[1] = o1;
-        } else {
-            const float sc = __bfloat162float(static_cast<const __nv_bfloat16*>(s)[(e * N + n) * (K / 128) + k0 / 128]);
-            const __nv_bfloat162 sc2 = __float2bfloat162_rn(sc);
-            dst[0] = decode_int4_8(raw.x, sc2);
-            dst[1] = decode_int4_8(raw.y, sc2);
-            dst[2] = decode_int4_8(raw.z, sc2);
-            dst[3] = decode_int4_8(raw.w, sc2);
+    uint4* dst = reinterpret_cast<uint4*>(out + e * N * (int64_t)K);
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t base = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; base < npieces; base += stride * kDqUnroll) {
+        uint2 raw[kDqUnroll];
+#pragma unroll
+        for (int u = 0; u < kDqUnroll; ++u) {
+            const int64_t pc = base + u * stride;
+            raw[u] = make_uint2(0, 0);
+            if (pc < npieces) {
+                if constexpr (kFp8) {
+                    raw[u] = __ldcs(reinterpret_cast<const uint2*>(src) + pc);
+                } else {
+                    raw[u].x = __ldcs(reinterpret_cast<const uint32_t*>(src) + pc);
+                }
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < kDqUnroll; ++u) {
+            const int64_t pc = base + u * stride;
+            if (pc >= npieces) break;
+            const int64_t elem = pc * 8;
+            const int n = (int)(elem / K);
+            const int k0 = (int)(elem - (int64_t)n * K);
+            if constexpr (kFp8) {
+                const float sc = static_cast<const float*>(s)[(e * (N / 128) + n / 128) * (K / 128) + k0 / 128];
+                uint4 o0, o1;  // decode_fp8_16 takes 16 bytes; the upper 8 are unused here
+                decode_fp8_16(make_uint4(raw[u].x, raw[u].y, 0, 0), sc, o0, o1);
+                dst[pc] = o0;
+            } else {
+                const float sc =
+                    __bfloat162float(static_cast<const __nv_bfloat16*>(s)[(e * N + n) * (K / 128) + k0 / 128]);
+                dst[pc] = decode_int4_8(raw[u].x, __float2bfloat162_rn(sc));
+            }
         }
     }
 }
@@ -743,8 +759,8 @@ static cudaError_t dequant_all(const FfnProblem& p, FfnProblem& q, cudaStream_t 
     const Part parts[3] = {{p.w_gate, p.s_gate, p.I, p.H, dq}, {p.w_up, p.s_up, p.I, p.H, dq + gu},
                            {p.w_down, p.s_down, p.H, p.I, dq + 2 * gu}};
     for (const Part& pt : parts) {
-        const int64_t nchunks = (int64_t)pt.N * pt.K / (p.w_dtype == GBMOE_FP8_E4M3_B128 ? 16 : 32);
-        const dim3 grid((unsigned)min64((nchunks + 1023) / 1024, 4096), (unsigned)p.E);
+        const int64_t npieces = (int64_t)pt.N * pt.K / 8;
+        const dim3 grid((unsigned)min64((npieces + 256 * kDqUnroll - 1) / (256 * kDqUnroll), 2048), (unsigned)p.E);
         if (p.w_dtype == GBMOE_FP8_E4M3_B128)
             dequant_weights_kernel<GBMOE_FP8_E4M3_B128><<<grid, 256, 0, stream>>>(
                 static_cast<const uint8_t*>(pt.w), pt.s, pt.N, pt.K, p.sched, pt.out);
