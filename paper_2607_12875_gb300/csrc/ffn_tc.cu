@@ -600,56 +600,57 @@ gather_rows_kernel(const uint4* __restrict__ x, const int32_t* __restrict__ sort
 
 // ------------------------------------- one-pass decode of quantised weights
 
-// Active experts' quantised [N, K] matrices -> bf16 [E, N, K]. A thread
-// decodes 8 consecutive weights at a time (8 fp8 bytes or one 32-bit word of
-// int4) into one 16-byte bf16 chunk, so a warp reads 256 or 128 contiguous
-// bytes and writes 512; each thread first loads kDqUnroll such pieces. The
-// decode functions and scale handling are the GEMM converter warps', so the
-// copy holds exactly the bf16 operands the in-GEMM decode would produce.
+// Active experts' quantised [N, K] matrices -> bf16 [E, N, K]. A warp takes
+// whole rows; lane l decodes the 8-weight pieces l, l+32, ... of the row (8
+// fp8 bytes or one 32-bit word of int4 each) into 16-byte bf16 chunks, so a
+// warp reads 256 or 128 contiguous bytes and writes 512 per step, with
+// kDqUnroll pieces loaded ahead. The decode functions and scale handling are
+// the GEMM converter warps', so the copy holds exactly the bf16 operands the
+// in-GEMM decode would produce.
 constexpr int kDqUnroll = 4;
+constexpr int kDqWarps = 8;
 
 template <int WQ>
-__global__ void __launch_bounds__(256)
+__global__ void __launch_bounds__(kDqWarps * 32)
 dequant_weights_kernel(const uint8_t* __restrict__ w, const void* __restrict__ s, int N, int K,
                        const int32_t* __restrict__ sched, __nv_bfloat16* __restrict__ out) {
     const int slot = blockIdx.y;
     if (slot >= sched[0]) return;
     const int64_t e = sched[kSchedHeader + slot];
     constexpr bool kFp8 = WQ == GBMOE_FP8_E4M3_B128;
-    const int64_t npieces = (int64_t)N * K / 8;  // 8 weights each
-    const uint8_t* src = w + e * N * (int64_t)(kFp8 ? K : K / 2);
-    uint4* dst = reinterpret_cast<uint4*>(out + e * N * (int64_t)K);
-    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t base = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; base < npieces; base += stride * kDqUnroll) {
-        uint2 raw[kDqUnroll];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int ppr = K / 8;      // pieces per row
+    const int kgroups = K / 128;
+    for (int n = blockIdx.x * kDqWarps + warp; n < N; n += gridDim.x * kDqWarps) {
+        const int64_t row = e * N + n;
+        const uint8_t* src = w + row * (kFp8 ? K : K / 2);
+        uint4* dst = reinterpret_cast<uint4*>(out + row * K);
+        // scale of 128-wide k group g of this row
+        const float* s8 = kFp8 ? static_cast<const float*>(s) + (e * (N / 128) + n / 128) * kgroups : nullptr;
+        const __nv_bfloat16* s4 = kFp8 ? nullptr : static_cast<const __nv_bfloat16*>(s) + row * kgroups;
+        for (int p0 = lane; p0 < ppr; p0 += 32 * kDqUnroll) {
+            uint2 raw[kDqUnroll];
 #pragma unroll
-        for (int u = 0; u < kDqUnroll; ++u) {
-            const int64_t pc = base + u * stride;
-            raw[u] = make_uint2(0, 0);
-            if (pc < npieces) {
-                if constexpr (kFp8) {
-                    raw[u] = __ldcs(reinterpret_cast<const uint2*>(src) + pc);
-                } else {
-                    raw[u].x = __ldcs(reinterpret_cast<const uint32_t*>(src) + pc);
+            for (int u = 0; u < kDqUnroll; ++u) {
+                const int pc = p0 + 32 * u;
+                raw[u] = make_uint2(0, 0);
+                if (pc < ppr) {
+                    if constexpr (kFp8) raw[u] = __ldcs(reinterpret_cast<const uint2*>(src) + pc);
+                    else raw[u].x = __ldcs(reinterpret_cast<const uint32_t*>(src) + pc);
                 }
             }
-        }
 #pragma unroll
-        for (int u = 0; u < kDqUnroll; ++u) {
-            const int64_t pc = base + u * stride;
-            if (pc >= npieces) break;
-            const int64_t elem = pc * 8;
-            const int n = (int)(elem / K);
-            const int k0 = (int)(elem - (int64_t)n * K);
-            if constexpr (kFp8) {
-                const float sc = static_cast<const float*>(s)[(e * (N / 128) + n / 128) * (K / 128) + k0 / 128];
-                uint4 o0, o1;  // decode_fp8_16 takes 16 bytes; the upper 8 are unused here
-                decode_fp8_16(make_uint4(raw[u].x, raw[u].y, 0, 0), sc, o0, o1);
-                dst[pc] = o0;
-            } else {
-                const float sc =
-                    __bfloat162float(static_cast<const __nv_bfloat16*>(s)[(e * N + n) * (K / 128) + k0 / 128]);
-                dst[pc] = decode_int4_8(raw[u].x, __float2bfloat162_rn(sc));
+            for (int u = 0; u < kDqUnroll; ++u) {
+                const int pc = p0 + 32 * u;
+                if (pc >= ppr) break;
+                const int g = pc >> 4;  // 16 pieces of 8 per 128-wide group
+                if constexpr (kFp8) {
+                    uint4 o0, o1;  // decode_fp8_16 takes 16 bytes; the upper 8 are unused here
+                    decode_fp8_16(make_uint4(raw[u].x, raw[u].y, 0, 0), s8[g], o0, o1);
+                    dst[pc] = o0;
+                } else {
+                    dst[pc] = decode_int4_8(raw[u].x, __float2bfloat162_rn(__bfloat162float(s4[g])));
+                }
             }
         }
     }
@@ -759,13 +760,12 @@ static cudaError_t dequant_all(const FfnProblem& p, FfnProblem& q, cudaStream_t 
     const Part parts[3] = {{p.w_gate, p.s_gate, p.I, p.H, dq}, {p.w_up, p.s_up, p.I, p.H, dq + gu},
                            {p.w_down, p.s_down, p.H, p.I, dq + 2 * gu}};
     for (const Part& pt : parts) {
-        const int64_t npieces = (int64_t)pt.N * pt.K / 8;
-        const dim3 grid((unsigned)min64((npieces + 256 * kDqUnroll - 1) / (256 * kDqUnroll), 2048), (unsigned)p.E);
+        const dim3 grid((unsigned)((pt.N + kDqWarps - 1) / kDqWarps), (unsigned)p.E);
         if (p.w_dtype == GBMOE_FP8_E4M3_B128)
-            dequant_weights_kernel<GBMOE_FP8_E4M3_B128><<<grid, 256, 0, stream>>>(
+            dequant_weights_kernel<GBMOE_FP8_E4M3_B128><<<grid, kDqWarps * 32, 0, stream>>>(
                 static_cast<const uint8_t*>(pt.w), pt.s, pt.N, pt.K, p.sched, pt.out);
         else
-            dequant_weights_kernel<GBMOE_INT4_G128><<<grid, 256, 0, stream>>>(
+            dequant_weights_kernel<GBMOE_INT4_G128><<<grid, kDqWarps * 32, 0, stream>>>(
                 static_cast<const uint8_t*>(pt.w), pt.s, pt.N, pt.K, p.sched, pt.out);
         const cudaError_t err = cudaGetLastError();
         if (err != cudaSuccess) return err;
