@@ -36,10 +36,15 @@ import synth  # noqa: E402
 METRIC = "MoE layer tokens/sec at 1 GB300; % of HBM (decode) / tensor-core (prefill) roofline"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
-# DRAM bytes per launch of the dominant kernel(s) from one ncu capture
-# (dram__bytes_read.sum + dram__bytes_write.sum), keyed by (workload, route);
-# absent (null) whenever the kernel changed since the counters were taken.
-TRAFFIC: dict = {}
+# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) of the expert-FFN
+# kernels per active expert, from one ncu capture of a reduced case with the
+# same H, I and dtypes (the streaming route reads each active expert's weights
+# once, so its traffic grows with the number of active experts); the bench
+# line reports it times this run's active experts. Keyed by (workload, route);
+# absent (null) whenever the kernels changed since the counters were taken.
+# decode: stream_gateup + stream_down on T=8, E=32 (29 active experts):
+# 730.0 + 3.4 + 365.2 + 3.0 MB.
+TRAFFIC_PER_ACTIVE_EXPERT: dict = {("decode_bf16_T32_H4096_E128_k8_I1536", "stream"): 1101.626e6 / 29}
 
 
 def peaks():
@@ -336,7 +341,8 @@ def main():
               "tc_dequant": "moe_grouped_ffn, tcgen05 decode-once route (3 weight-decode passes + row gather + "
                             "gate/up GEMM with SwiGLU + down GEMM)",
               "simt": "moe_grouped_ffn, CUDA-core route"}[route]
-    common = {"traffic": TRAFFIC.get((wl.name, route)), "kernel": kernel, "algorithmic_bytes": routed_bytes,
+    tpe = TRAFFIC_PER_ACTIVE_EXPERT.get((wl.name, route))
+    common = {"traffic": None if tpe is None else tpe * active, "kernel": kernel, "algorithmic_bytes": routed_bytes,
               "algorithmic_flops": flops, "active_experts": active, "ms_per_launch": ffn_ms,
               "roofline_ms": max(t_hbm, t_tensor) * 1e3}
     if t_hbm >= t_tensor:
