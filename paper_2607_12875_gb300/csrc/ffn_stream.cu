@@ -10,7 +10,8 @@
 // each activation chunk once and decodes the weights per activation row, so
 // the kernel stays within 128 registers and two CTAs (16 warps) share an SM.
 // Up to kNT rows are handled per weight pass; more rows take further passes
-// over the same weights.
+// over the same weights. A CTA covers up to 4 column groups in turn, so it
+// stages its activation rows once for all of them.
 //   stage 1: h[r, i] = silu(x_r . Wgate[i]) * (x_r . Wup[i]), 2 columns per warp
 //   stage 2: y[r, n] = h_r . Wdown[n], 4 output columns per warp
 #include <type_traits>
@@ -25,6 +26,8 @@ namespace gbmoe {
 constexpr int kStreamWarps = 8;
 constexpr int kNT = 8;      // activation rows per weight pass
 constexpr int kUnroll = 4;  // chunks per row loaded before use
+constexpr int kMaxGroupsPerCta = 4;
+constexpr int kMinWaves = 8;
 
 // CTAs per SM the register budget is set for: two for bf16 weights (the
 // decode path); fp32 and quantised weights hold or decode more per element
@@ -114,9 +117,43 @@ __device__ __forceinline__ void dispatch_nt(int nt, F&& f) {
     else f(std::integral_constant<int, 8>{});
 }
 
-template <typename TA, int WQ>
-__global__ void __launch_bounds__(kStreamWarps * 32, stream_min_blocks<WQ>())
-stream_gateup_kernel(FfnProblem p) {
+// Weight rows of column group g: 2 gate + 2 up rows (stage 1) or 4 down rows
+// (stage 2) per warp, with their scale rows; col0 = first output column.
+template <int WQ, int STAGE>
+__device__ __forceinline__ void group_rows(const FfnProblem& p, int e, int g, int warp, const uint8_t* (&wrow)[4],
+                                           const void* (&srow)[4], int& col0) {
+    using F = WFmt<WQ>;
+    const int H = p.H, I = p.I;
+    if (STAGE == 1) {
+        const size_t rb = F::row_bytes(H);
+        const int i0 = (g * kStreamWarps + warp) * 2;
+        const uint8_t* wg = static_cast<const uint8_t*>(p.w_gate) + (size_t)e * I * rb;
+        const uint8_t* wu = static_cast<const uint8_t*>(p.w_up) + (size_t)e * I * rb;
+        wrow[0] = wg + i0 * rb; wrow[1] = wg + (i0 + 1) * rb; wrow[2] = wu + i0 * rb; wrow[3] = wu + (i0 + 1) * rb;
+        srow[0] = F::scale_row(p.s_gate, e, I, H, i0); srow[1] = F::scale_row(p.s_gate, e, I, H, i0 + 1);
+        srow[2] = F::scale_row(p.s_up, e, I, H, i0); srow[3] = F::scale_row(p.s_up, e, I, H, i0 + 1);
+        col0 = i0;
+    } else {
+        const size_t rb = F::row_bytes(I);
+        const int n0 = (g * kStreamWarps + warp) * 4;
+        const uint8_t* wd = static_cast<const uint8_t*>(p.w_down) + (size_t)e * H * rb;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            wrow[q] = wd + (n0 + q) * rb;
+            srow[q] = F::scale_row(p.s_down, e, H, I, n0 + q);
+        }
+        col0 = n0;
+    }
+}
+
+// One CTA: one active expert and gpc consecutive column groups (a group is 8
+// warps x 2 h-columns in stage 1, 8 warps x 4 y-columns in stage 2). The
+// expert's activation rows are staged once per pass of kNT rows and serve
+// all of the CTA's groups.
+//   stage 1: h[r, i] = silu(x_r . Wgate[i]) * (x_r . Wup[i])
+//   stage 2: y[r, n] = h_r . Wdown[n]
+template <typename TA, int WQ, int STAGE>
+__device__ __forceinline__ void stream_ffn_cta(const FfnProblem& p, int gpc) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     TA* xs = reinterpret_cast<TA*>(smem_raw);
     const int slot = blockIdx.x;
@@ -125,84 +162,70 @@ stream_gateup_kernel(FfnProblem p) {
     const int64_t cnt = p.counts ? p.counts[e] : p.n_rows;
     const int64_t row0 = p.offsets ? p.offsets[e] : 0;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int i0 = (blockIdx.y * kStreamWarps + warp) * 2;
-    const int H = p.H, I = p.I;
-    using F = WFmt<WQ>;
-    const size_t rb = F::row_bytes(H);
-    const uint8_t* wg = static_cast<const uint8_t*>(p.w_gate) + (size_t)e * I * rb;
-    const uint8_t* wu = static_cast<const uint8_t*>(p.w_up) + (size_t)e * I * rb;
-    const uint8_t* const wrow[4] = {wg + i0 * rb, wg + (i0 + 1) * rb, wu + i0 * rb, wu + (i0 + 1) * rb};
-    const void* const srow[4] = {F::scale_row(p.s_gate, e, I, H, i0), F::scale_row(p.s_gate, e, I, H, i0 + 1),
-                                 F::scale_row(p.s_up, e, I, H, i0), F::scale_row(p.s_up, e, I, H, i0 + 1)};
-    TA* h = static_cast<TA*>(p.h);
+    const int K = STAGE == 1 ? p.H : p.I;
+    TA* out = static_cast<TA*>(STAGE == 1 ? p.h : p.y);
+    const int out_cols = STAGE == 1 ? p.I : p.H;
     for (int64_t p0 = 0; p0 < cnt; p0 += kNT) {
         const int nt = (int)min64(kNT, cnt - p0);
         __syncthreads();
-        stage_rows<TA>(xs, static_cast<const TA*>(p.x), H, p.sorted_pair, p.pair_div, row0 + p0, nt);
+        if (STAGE == 1) stage_rows<TA>(xs, static_cast<const TA*>(p.x), K, p.sorted_pair, p.pair_div, row0 + p0, nt);
+        else stage_rows<TA>(xs, static_cast<const TA*>(p.h), K, nullptr, 1, row0 + p0, nt);
         __syncthreads();
         dispatch_nt(nt, [&](auto NTc) {
             constexpr int NT = decltype(NTc)::value;
-            float acc[4][NT];
+#pragma unroll 1
+            for (int g = blockIdx.y * gpc; g < (blockIdx.y + 1) * gpc; ++g) {
+                const uint8_t* wrow[4];
+                const void* srow[4];
+                int col0;
+                group_rows<WQ, STAGE>(p, e, g, warp, wrow, srow, col0);
+                float acc[4][NT];
 #pragma unroll
-            for (int q = 0; q < 4; ++q)
+                for (int q = 0; q < 4; ++q)
 #pragma unroll
-                for (int r = 0; r < NT; ++r) acc[q][r] = 0.0f;
-            dot4<TA, WQ, NT>(wrow, srow, xs, H, acc);
-            warp_sum<NT>(acc);
+                    for (int r = 0; r < NT; ++r) acc[q][r] = 0.0f;
+                dot4<TA, WQ, NT>(wrow, srow, xs, K, acc);
+                warp_sum<NT>(acc);
 #pragma unroll
-            for (int r = 0; r < NT; ++r)
-                if (r == lane && r < nt) {
-                    TA* dst = h + (row0 + p0 + r) * I + i0;
-                    dst[0] = from_f32<TA>(silu_mul(acc[0][r], acc[2][r]));
-                    dst[1] = from_f32<TA>(silu_mul(acc[1][r], acc[3][r]));
-                }
+                for (int r = 0; r < NT; ++r)
+                    if (r == lane && r < nt) {
+                        TA* dst = out + (row0 + p0 + r) * out_cols + col0;
+                        if (STAGE == 1) {
+                            dst[0] = from_f32<TA>(silu_mul(acc[0][r], acc[2][r]));
+                            dst[1] = from_f32<TA>(silu_mul(acc[1][r], acc[3][r]));
+                        } else {
+#pragma unroll
+                            for (int q = 0; q < 4; ++q) dst[q] = from_f32<TA>(acc[q][r]);
+                        }
+                    }
+            }
         });
     }
 }
 
 template <typename TA, int WQ>
 __global__ void __launch_bounds__(kStreamWarps * 32, stream_min_blocks<WQ>())
-stream_down_kernel(FfnProblem p) {
-    extern __shared__ __align__(16) unsigned char smem_raw[];
-    TA* hs = reinterpret_cast<TA*>(smem_raw);
-    const int slot = blockIdx.x;
-    if (slot >= p.sched[0]) return;
-    const int e = p.sched[kSchedHeader + slot];
-    const int64_t cnt = p.counts ? p.counts[e] : p.n_rows;
-    const int64_t row0 = p.offsets ? p.offsets[e] : 0;
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int n0 = (blockIdx.y * kStreamWarps + warp) * 4;
-    const int H = p.H, I = p.I;
-    using F = WFmt<WQ>;
-    const size_t rb = F::row_bytes(I);
-    const uint8_t* wd = static_cast<const uint8_t*>(p.w_down) + (size_t)e * H * rb;
-    const uint8_t* const wrow[4] = {wd + n0 * rb, wd + (n0 + 1) * rb, wd + (n0 + 2) * rb, wd + (n0 + 3) * rb};
-    const void* const srow[4] = {F::scale_row(p.s_down, e, H, I, n0), F::scale_row(p.s_down, e, H, I, n0 + 1),
-                                 F::scale_row(p.s_down, e, H, I, n0 + 2), F::scale_row(p.s_down, e, H, I, n0 + 3)};
-    TA* y = static_cast<TA*>(p.y);
-    for (int64_t p0 = 0; p0 < cnt; p0 += kNT) {
-        const int nt = (int)min64(kNT, cnt - p0);
-        __syncthreads();
-        stage_rows<TA>(hs, static_cast<const TA*>(p.h), I, nullptr, 1, row0 + p0, nt);
-        __syncthreads();
-        dispatch_nt(nt, [&](auto NTc) {
-            constexpr int NT = decltype(NTc)::value;
-            float acc[4][NT];
-#pragma unroll
-            for (int q = 0; q < 4; ++q)
-#pragma unroll
-                for (int r = 0; r < NT; ++r) acc[q][r] = 0.0f;
-            dot4<TA, WQ, NT>(wrow, srow, hs, I, acc);
-            warp_sum<NT>(acc);
-#pragma unroll
-            for (int r = 0; r < NT; ++r)
-                if (r == lane && r < nt) {
-                    TA* dst = y + (row0 + p0 + r) * H + n0;
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) dst[q] = from_f32<TA>(acc[q][r]);
-                }
-        });
-    }
+stream_gateup_kernel(FfnProblem p, int gpc) {
+    stream_ffn_cta<TA, WQ, 1>(p, gpc);
+}
+
+template <typename TA, int WQ>
+__global__ void __launch_bounds__(kStreamWarps * 32, stream_min_blocks<WQ>())
+stream_down_kernel(FfnProblem p, int gpc) {
+    stream_ffn_cta<TA, WQ, 2>(p, gpc);
+}
+
+// Column groups per CTA: up to kMaxGroupsPerCta while the grid keeps at least
+// kMinWaves waves of CTAs (fewer, longer CTAs stage the rows less often;
+// too few CTAs leave SMs idle). groups is a multiple of 8.
+static int groups_per_cta(int max_active, int groups) {
+    int sms = 0, dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int64_t slots = (int64_t)(sms > 0 ? sms : 1) * 2;  // resident CTAs (two per SM)
+    int gpc = kMaxGroupsPerCta;
+    while (gpc > 1 && (int64_t)max_active * (groups / gpc) < kMinWaves * slots) gpc /= 2;
+    return gpc;
 }
 
 template <typename TA, int WQ>
@@ -216,11 +239,13 @@ static cudaError_t launch_stream_t(const FfnProblem& p, cudaStream_t stream) {
     if (err != cudaSuccess) return err;
     err = cudaFuncSetAttribute(stream_down_kernel<TA, WQ>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem2);
     if (err != cudaSuccess) return err;
-    dim3 g1(max_active, p.I / (2 * kStreamWarps));
-    stream_gateup_kernel<TA, WQ><<<g1, kStreamWarps * 32, smem1, stream>>>(p);
+    const int groups1 = p.I / (2 * kStreamWarps), groups2 = p.H / (4 * kStreamWarps);
+    const int gpc1 = groups_per_cta(max_active, groups1), gpc2 = groups_per_cta(max_active, groups2);
+    dim3 g1(max_active, groups1 / gpc1);
+    stream_gateup_kernel<TA, WQ><<<g1, kStreamWarps * 32, smem1, stream>>>(p, gpc1);
     if ((err = cudaGetLastError()) != cudaSuccess) return err;
-    dim3 g2(max_active, p.H / (4 * kStreamWarps));
-    stream_down_kernel<TA, WQ><<<g2, kStreamWarps * 32, smem2, stream>>>(p);
+    dim3 g2(max_active, groups2 / gpc2);
+    stream_down_kernel<TA, WQ><<<g2, kStreamWarps * 32, smem2, stream>>>(p, gpc2);
     return cudaGetLastError();
 }
 
