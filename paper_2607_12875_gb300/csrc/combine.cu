@@ -10,6 +10,7 @@ template <typename TA>
 __global__ void __launch_bounds__(256)
 combine_kernel(const TA* __restrict__ y, const float* __restrict__ w, const int32_t* __restrict__ pair_pos,
                const TA* __restrict__ y_shared, TA* __restrict__ out, int k, int H) {
+    pdl_enter();
     const int t = blockIdx.x;
     __shared__ int32_t s_pos[32];
     __shared__ float s_w[32];
@@ -41,14 +42,11 @@ cudaError_t launch_combine(const void* y_pairs, const float* topk_w, const int32
                            void* out, int T, int k, int H, int act_dtype, cudaStream_t stream) {
     if (T == 0) return cudaSuccess;
     if (act_dtype == GBMOE_BF16)
-        combine_kernel<__nv_bfloat16><<<T, 256, 0, stream>>>(
-            static_cast<const __nv_bfloat16*>(y_pairs), topk_w, pair_pos,
-            static_cast<const __nv_bfloat16*>(y_shared), static_cast<__nv_bfloat16*>(out), k, H);
-    else
-        combine_kernel<float><<<T, 256, 0, stream>>>(static_cast<const float*>(y_pairs), topk_w, pair_pos,
-                                                     static_cast<const float*>(y_shared),
-                                                     static_cast<float*>(out), k, H);
-    return cudaGetLastError();
+        return launch_k(combine_kernel<__nv_bfloat16>, dim3(T), dim3(256), 0, stream,
+                        static_cast<const __nv_bfloat16*>(y_pairs), topk_w, pair_pos,
+                        static_cast<const __nv_bfloat16*>(y_shared), static_cast<__nv_bfloat16*>(out), k, H);
+    return launch_k(combine_kernel<float>, dim3(T), dim3(256), 0, stream, static_cast<const float*>(y_pairs), topk_w,
+                    pair_pos, static_cast<const float*>(y_shared), static_cast<float*>(out), k, H);
 }
 
 }  // namespace gbmoe

@@ -13,6 +13,7 @@ size_t ffn_sched_ints(int E, int64_t n_rows) {
 
 __global__ void __launch_bounds__(512)
 ffn_schedule_kernel(const int32_t* __restrict__ counts, int E, int64_t n_rows, int BM, int32_t* __restrict__ sched) {
+    pdl_enter();
     __shared__ int32_t s_warp_t[16], s_warp_a[16];
     const int e = threadIdx.x, lane = e & 31, warp = e >> 5;
     int cnt = 0;
@@ -55,7 +56,9 @@ ffn_schedule_kernel(const int32_t* __restrict__ counts, int E, int64_t n_rows, i
 
 cudaError_t launch_ffn_schedule(const int32_t* counts, int E, int64_t n_rows, int BM, int32_t* sched,
                                 cudaStream_t stream) {
-    ffn_schedule_kernel<<<1, 512, 0, stream>>>(counts, E, n_rows, BM, sched);
+    if (const cudaError_t le = launch_k(ffn_schedule_kernel, dim3(1), dim3(512), 0, stream, counts, E, n_rows, BM,
+            sched); le != cudaSuccess)
+        return le;
     return cudaGetLastError();
 }
 

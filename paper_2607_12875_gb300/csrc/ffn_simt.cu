@@ -18,6 +18,7 @@ static_assert(kBM == kSchedMinBM, "tile list is built for the SIMT tile height")
 template <typename TA, int WQ>
 __global__ void __launch_bounds__(256)
 simt_gateup_kernel(FfnProblem p) {
+    pdl_enter();
     __shared__ float As[kBM][kBK + 1];
     __shared__ float Bg[kBN][kBK + 1];
     __shared__ float Bu[kBN][kBK + 1];
@@ -74,6 +75,7 @@ simt_gateup_kernel(FfnProblem p) {
 template <typename TA, int WQ>
 __global__ void __launch_bounds__(256)
 simt_down_kernel(FfnProblem p) {
+    pdl_enter();
     __shared__ float As[kBM][kBK + 1];
     __shared__ float Bd[kBN][kBK + 1];
     const int32_t* sched = p.sched;
@@ -120,11 +122,13 @@ static cudaError_t launch_simt_t(const FfnProblem& p, cudaStream_t stream) {
     const int64_t max_tiles = sched_max_tiles(p.E, p.n_rows, kBM);
     if (p.n_rows == 0) return cudaSuccess;
     dim3 g1((unsigned)max_tiles, p.I / kBN);
-    simt_gateup_kernel<TA, WQ><<<g1, 256, 0, stream>>>(p);
+    if (const cudaError_t le = launch_k(simt_gateup_kernel<TA, WQ>, dim3(g1), dim3(256), 0, stream, p); le != cudaSuccess)
+        return le;
     cudaError_t err = cudaGetLastError();
     if (err != cudaSuccess) return err;
     dim3 g2((unsigned)max_tiles, p.H / kBN);
-    simt_down_kernel<TA, WQ><<<g2, 256, 0, stream>>>(p);
+    if (const cudaError_t le = launch_k(simt_down_kernel<TA, WQ>, dim3(g2), dim3(256), 0, stream, p); le != cudaSuccess)
+        return le;
     return cudaGetLastError();
 }
 

@@ -206,12 +206,14 @@ __device__ __forceinline__ void stream_ffn_cta(const FfnProblem& p, int gpc) {
 template <typename TA, int WQ>
 __global__ void __launch_bounds__(kStreamWarps * 32, stream_min_blocks<WQ>())
 stream_gateup_kernel(FfnProblem p, int gpc) {
+    pdl_enter();
     stream_ffn_cta<TA, WQ, 1>(p, gpc);
 }
 
 template <typename TA, int WQ>
 __global__ void __launch_bounds__(kStreamWarps * 32, stream_min_blocks<WQ>())
 stream_down_kernel(FfnProblem p, int gpc) {
+    pdl_enter();
     stream_ffn_cta<TA, WQ, 2>(p, gpc);
 }
 
@@ -242,10 +244,14 @@ static cudaError_t launch_stream_t(const FfnProblem& p, cudaStream_t stream) {
     const int groups1 = p.I / (2 * kStreamWarps), groups2 = p.H / (4 * kStreamWarps);
     const int gpc1 = groups_per_cta(max_active, groups1), gpc2 = groups_per_cta(max_active, groups2);
     dim3 g1(max_active, groups1 / gpc1);
-    stream_gateup_kernel<TA, WQ><<<g1, kStreamWarps * 32, smem1, stream>>>(p, gpc1);
+    if (const cudaError_t le = launch_k(stream_gateup_kernel<TA, WQ>, dim3(g1), dim3(kStreamWarps * 32), smem1,
+            stream, p, gpc1); le != cudaSuccess)
+        return le;
     if ((err = cudaGetLastError()) != cudaSuccess) return err;
     dim3 g2(max_active, groups2 / gpc2);
-    stream_down_kernel<TA, WQ><<<g2, kStreamWarps * 32, smem2, stream>>>(p, gpc2);
+    if (const cudaError_t le = launch_k(stream_down_kernel<TA, WQ>, dim3(g2), dim3(kStreamWarps * 32), smem2,
+            stream, p, gpc2); le != cudaSuccess)
+        return le;
     return cudaGetLastError();
 }
 

@@ -337,6 +337,7 @@ template <int WQ>
 __global__ void __launch_bounds__(Fmt<WQ>::THREADS, 1)
 tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b0,
                const __grid_constant__ CUtensorMap tm_b1, const __grid_constant__ CUtensorMap tm_out, const Params p) {
+    pdl_enter();
     using L = Layout<WQ>;
     constexpr int STAGES = L::STAGES;
     constexpr int RAW = Fmt<WQ>::RAW_BYTES;
@@ -589,6 +590,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
 __global__ void __launch_bounds__(256)
 gather_rows_kernel(const uint4* __restrict__ x, const int32_t* __restrict__ sorted_pair, int pair_div,
                    int64_t n_rows, int vec_per_row, uint4* __restrict__ out) {
+    pdl_enter();
     const int64_t total = n_rows * vec_per_row;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
         const int64_t r = i / vec_per_row;
@@ -614,6 +616,7 @@ template <int WQ>
 __global__ void __launch_bounds__(kDqWarps * 32)
 dequant_weights_kernel(const uint8_t* __restrict__ w, const void* __restrict__ s, int N, int K,
                        const int32_t* __restrict__ sched, __nv_bfloat16* __restrict__ out) {
+    pdl_enter();
     const int slot = blockIdx.y;
     if (slot >= sched[0]) return;
     const int64_t e = sched[kSchedHeader + slot];
@@ -727,7 +730,9 @@ static cudaError_t launch_gemm_t(const CUtensorMap& a, const CUtensorMap& b0, co
     if (e != cudaSuccess) return e;
     const int grid = (int)min64(num_sms(), max_work);
     if (grid <= 0) return cudaSuccess;
-    tc_gemm_kernel<WQ><<<grid, Fmt<WQ>::THREADS, Layout<WQ>::SMEM_BYTES, stream>>>(a, b0, b1, out, prm);
+    if (const cudaError_t le = launch_k(tc_gemm_kernel<WQ>, dim3(grid), dim3(Fmt<WQ>::THREADS),
+            Layout<WQ>::SMEM_BYTES, stream, a, b0, b1, out, prm); le != cudaSuccess)
+        return le;
     return cudaGetLastError();
 }
 
@@ -761,13 +766,12 @@ static cudaError_t dequant_all(const FfnProblem& p, FfnProblem& q, cudaStream_t 
                            {p.w_down, p.s_down, p.H, p.I, dq + 2 * gu}};
     for (const Part& pt : parts) {
         const dim3 grid((unsigned)((pt.N + kDqWarps - 1) / kDqWarps), (unsigned)p.E);
-        if (p.w_dtype == GBMOE_FP8_E4M3_B128)
-            dequant_weights_kernel<GBMOE_FP8_E4M3_B128><<<grid, kDqWarps * 32, 0, stream>>>(
-                static_cast<const uint8_t*>(pt.w), pt.s, pt.N, pt.K, p.sched, pt.out);
-        else
-            dequant_weights_kernel<GBMOE_INT4_G128><<<grid, kDqWarps * 32, 0, stream>>>(
-                static_cast<const uint8_t*>(pt.w), pt.s, pt.N, pt.K, p.sched, pt.out);
-        const cudaError_t err = cudaGetLastError();
+        const cudaError_t err =
+            p.w_dtype == GBMOE_FP8_E4M3_B128
+                ? launch_k(dequant_weights_kernel<GBMOE_FP8_E4M3_B128>, dim3(grid), dim3(kDqWarps * 32), 0, stream,
+                           static_cast<const uint8_t*>(pt.w), pt.s, pt.N, pt.K, p.sched, pt.out)
+                : launch_k(dequant_weights_kernel<GBMOE_INT4_G128>, dim3(grid), dim3(kDqWarps * 32), 0, stream,
+                           static_cast<const uint8_t*>(pt.w), pt.s, pt.N, pt.K, p.sched, pt.out);
         if (err != cudaSuccess) return err;
     }
     q.w_dtype = GBMOE_BF16;
@@ -792,8 +796,10 @@ cudaError_t launch_ffn_tc(const FfnProblem& pin, cudaStream_t stream) {
         const int vpr = p.H * 2 / 16;
         const int64_t nvec = p.n_rows * vpr;
         const int gblocks = (int)min64((nvec + 255) / 256, 152 * 16);
-        gather_rows_kernel<<<gblocks, 256, 0, stream>>>(static_cast<const uint4*>(p.x), p.sorted_pair, p.pair_div,
-                                                        p.n_rows, vpr, static_cast<uint4*>(p.x_sorted));
+        if (const cudaError_t le = launch_k(gather_rows_kernel, dim3(gblocks), dim3(256), 0, stream,
+                static_cast<const uint4*>(p.x), p.sorted_pair, p.pair_div, p.n_rows, vpr,
+                static_cast<uint4*>(p.x_sorted)); le != cudaSuccess)
+            return le;
         if ((err = cudaGetLastError()) != cudaSuccess) return err;
         a_rows = p.x_sorted;
     }

@@ -17,6 +17,7 @@ size_t permute_scratch_ints(int64_t P, int E) { return 2 * (size_t)permute_block
 
 __global__ void __launch_bounds__(kPermBlock)
 perm_hist_kernel(const int32_t* __restrict__ ids, int64_t P, int E, int32_t* __restrict__ block_hist) {
+    pdl_enter();
     extern __shared__ int32_t s_hist[];
     for (int e = threadIdx.x; e < E; e += blockDim.x) s_hist[e] = 0;
     __syncthreads();
@@ -33,6 +34,7 @@ perm_hist_kernel(const int32_t* __restrict__ ids, int64_t P, int E, int32_t* __r
 __global__ void __launch_bounds__(512)
 perm_scan_kernel(const int32_t* __restrict__ block_hist, int nblk, int E, int32_t* __restrict__ counts,
                  int32_t* __restrict__ offsets, int32_t* __restrict__ block_base) {
+    pdl_enter();
     __shared__ int32_t s_warp[16];
     const int e = threadIdx.x;
     int run = 0;
@@ -73,6 +75,7 @@ perm_scan_kernel(const int32_t* __restrict__ block_hist, int nblk, int E, int32_
 __global__ void __launch_bounds__(kPermBlock)
 perm_scatter_kernel(const int32_t* __restrict__ ids, int64_t P, int E, const int32_t* __restrict__ block_base,
                     int32_t* __restrict__ sorted_pair, int32_t* __restrict__ pair_pos) {
+    pdl_enter();
     extern __shared__ int32_t s_run[];
     for (int e = threadIdx.x; e < E; e += blockDim.x) s_run[e] = block_base[(size_t)blockIdx.x * E + e];
     __syncthreads();
@@ -106,15 +109,20 @@ cudaError_t launch_permute(const int32_t* topk_ids, int64_t P, int E, int32_t* c
     int32_t* block_hist = scratch;
     int32_t* block_base = scratch + (size_t)nblk * E;
     if (nblk > 0) {
-        perm_hist_kernel<<<nblk, kPermBlock, E * sizeof(int32_t), stream>>>(topk_ids, P, E, block_hist);
+        if (const cudaError_t le = launch_k(perm_hist_kernel, dim3(nblk), dim3(kPermBlock), E * sizeof(int32_t),
+                stream, topk_ids, P, E, block_hist); le != cudaSuccess)
+            return le;
         cudaError_t err = cudaGetLastError();
         if (err != cudaSuccess) return err;
     }
-    perm_scan_kernel<<<1, 512, 0, stream>>>(block_hist, nblk, E, counts, offsets, block_base);
+    if (const cudaError_t le = launch_k(perm_scan_kernel, dim3(1), dim3(512), 0, stream, block_hist, nblk, E,
+            counts, offsets, block_base); le != cudaSuccess)
+        return le;
     cudaError_t err = cudaGetLastError();
     if (err != cudaSuccess || nblk == 0) return err;
-    perm_scatter_kernel<<<nblk, kPermBlock, E * sizeof(int32_t), stream>>>(topk_ids, P, E, block_base,
-                                                                           sorted_pair, pair_pos);
+    if (const cudaError_t le = launch_k(perm_scatter_kernel, dim3(nblk), dim3(kPermBlock), E * sizeof(int32_t),
+            stream, topk_ids, P, E, block_base, sorted_pair, pair_pos); le != cudaSuccess)
+        return le;
     return cudaGetLastError();
 }
 

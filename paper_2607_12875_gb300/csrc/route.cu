@@ -20,6 +20,7 @@ template <typename TA, int TB>
 __global__ void __launch_bounds__(kGateWarps * 32)
 gate_logits_kernel(const TA* __restrict__ x, const TA* __restrict__ wg, const float* __restrict__ bias,
                    float* __restrict__ logits, int T, int H, int E) {
+    pdl_enter();
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int t0 = blockIdx.x * TB;
     const int e0 = (blockIdx.y * kGateWarps + warp) * kGateExpertsPerWarp;
@@ -100,6 +101,7 @@ __device__ __forceinline__ void cp_async16(void* dst, const void* src, bool vali
 __global__ void __launch_bounds__(256, 1)
 gate_logits_tiled_kernel(const __nv_bfloat16* __restrict__ x, const __nv_bfloat16* __restrict__ wg,
                          const float* __restrict__ bias, float* __restrict__ logits, int T, int H, int E) {
+    pdl_enter();
     extern __shared__ __align__(16) uint8_t smem[];
     uint8_t* sx = smem;                                          // [stage][kGT][kSlab] bf16
     uint8_t* sw = smem + (size_t)kGStages * kGT * kSlab * 2;     // [stage][kGE][kSlab] bf16
@@ -243,6 +245,7 @@ constexpr int kMaxE = 512;
 __global__ void __launch_bounds__(kSelWarps * 32)
 select_experts_kernel(const float* __restrict__ logits, const float* __restrict__ select_bias,
                       int32_t* __restrict__ topk_ids, float* __restrict__ topk_w, RouteParams rp) {
+    pdl_enter();
     __shared__ float s_key[kSelWarps][kMaxE];
     __shared__ float s_sig[kSelWarps][kMaxE];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -354,23 +357,28 @@ cudaError_t launch_route(const RouteParams& rp, const void* x, const void* wg, c
                                                  (int)kGateTiledSmem);
             if (e != cudaSuccess) return e;
             dim3 grid((rp.T + kGT - 1) / kGT, (rp.E + kGE - 1) / kGE);
-            gate_logits_tiled_kernel<<<grid, 256, kGateTiledSmem, stream>>>(xp, wp, logit_bias, logits, rp.T, rp.H,
-                                                                            rp.E);
+            if (const cudaError_t le = launch_k(gate_logits_tiled_kernel, dim3(grid), dim3(256), kGateTiledSmem,
+                    stream, xp, wp, logit_bias, logits, rp.T, rp.H, rp.E); le != cudaSuccess)
+                return le;
         } else {
             dim3 grid((rp.T + 1) / 2, ey);
-            gate_logits_kernel<__nv_bfloat16, 2><<<grid, block, 0, stream>>>(xp, wp, logit_bias, logits, rp.T,
-                                                                              rp.H, rp.E);
+            if (const cudaError_t le = launch_k(gate_logits_kernel<__nv_bfloat16, 2>, dim3(grid), dim3(block), 0,
+                    stream, xp, wp, logit_bias, logits, rp.T, rp.H, rp.E); le != cudaSuccess)
+                return le;
         }
     } else {
         auto xp = static_cast<const float*>(x);
         auto wp = static_cast<const float*>(wg);
         dim3 grid((rp.T + 1) / 2, ey);
-        gate_logits_kernel<float, 2><<<grid, block, 0, stream>>>(xp, wp, logit_bias, logits, rp.T, rp.H, rp.E);
+        if (const cudaError_t le = launch_k(gate_logits_kernel<float, 2>, dim3(grid), dim3(block), 0, stream, xp,
+                wp, logit_bias, logits, rp.T, rp.H, rp.E); le != cudaSuccess)
+            return le;
     }
     cudaError_t err = cudaGetLastError();
     if (err != cudaSuccess) return err;
-    select_experts_kernel<<<(rp.T + kSelWarps - 1) / kSelWarps, kSelWarps * 32, 0, stream>>>(
-        logits, select_bias, topk_ids, topk_w, rp);
+    if (const cudaError_t le = launch_k(select_experts_kernel, dim3((rp.T + kSelWarps - 1) / kSelWarps),
+            dim3(kSelWarps * 32), 0, stream, logits, select_bias, topk_ids, topk_w, rp); le != cudaSuccess)
+        return le;
     return cudaGetLastError();
 }
 
