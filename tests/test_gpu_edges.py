@@ -128,3 +128,24 @@ def test_large_batch_routing_is_bit_exact(T, E, k, H):
     ref_ids, ref_w = oracle.route(oracle.gate_logits(x32, g32), k)
     assert np.array_equal(ids.cpu().numpy(), ref_ids)
     np.testing.assert_allclose(w.cpu().numpy(), ref_w, rtol=2e-6, atol=1e-7)
+
+
+# The streaming kernels let one CTA cover 1, 2 or 4 column groups, as many as
+# keep 8 waves of CTAs (two per SM) in the grid. The decode workload itself
+# takes 4; these shapes take 2 (64 active experts) and 4 with more rows per
+# expert than one pass over the weights holds (16 rows, kNT = 8).
+DECODE = synth.WORKLOADS[2]
+
+
+@pytest.mark.parametrize("T,E,k", [(8, 64, 8), (256, 128, 8)])
+def test_streaming_column_groups_per_cta(T, E, k):
+    wl = DECODE.replace(T=T, E=E, top_k=k, seed=90 + T)
+    assert wl.P <= 16 * wl.E  # streaming route
+    inp, out, ids, counts = run(wl, "stream")
+    rows = np.unique(np.r_[np.arange(min(T, 24)), np.arange(T - 8, T)]) if T > 32 else None
+    ref = oracle.forward(wl, inp, rows=rows)
+    assert np.array_equal(ids.cpu().numpy(), ref["topk_ids"])
+    assert np.array_equal(counts.cpu().numpy(), ref["counts"])
+    got = act_np(out) if rows is None else act_np(out)[ref["rows"]]
+    err = rel_err(got, ref["out"])
+    assert err <= tol_for(wl), f"rel err {err:.3e}"
