@@ -15,17 +15,21 @@
 //             16-wide slice, releasing ring slots and accumulators through
 //             tcgen05.commit -> mbarrier;
 //   warps 2-5 read the accumulator with tcgen05.ld (warp w owns TMEM lanes
-//             32*(w%4)..+31, i.e. tile rows) and write bf16 results:
+//             32*(w%4)..+31, i.e. tile rows) and produce bf16 results:
 //             h = silu(gate) * up for the gate/up GEMM (B rows 0-127 are the
 //             gate rows, 128-255 the up rows of the same 128 columns), plain
-//             y for the down GEMM.
+//             y for the down GEMM; each warp stages 32 rows x 32 columns in
+//             shared memory and writes them with one TMA store.
 // Quantised weights (fp8 e4m3 with 128x128 block scales, int4 with 128-wide
 // group scales) take the same path with eight more warps: TMA brings the raw
 // weight tile (64- or 32-byte swizzled rows) next to the A tile, and
 // warps 6-13, one B row per thread, decode it, apply the scale and write
 // the bf16 operand in the 128-byte-swizzled layout the MMA reads, then
-// signal the MMA warp. Decoding inside the kernel means no dequantised copy
-// of the weights ever exists in HBM.
+// signal the MMA warp. This keeps quantised weights quantised in HBM. When
+// experts have many rows, so that several M tiles would decode the same
+// weight tile again, the caller's workspace instead receives one bf16 copy
+// of the active experts' weights (dequant_weights_kernel, same decode) and
+// the bf16 GEMM runs on it.
 // Every mbarrier wait is bounded (about two seconds); on expiry the CTA sets
 // the device error word, stops issuing work, drains what it issued and
 // frees its TMEM.
