@@ -389,13 +389,17 @@ def main():
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         import oracle
 
+        # the first 32 tokens, repeated until about 10 s of oracle work (at most 8 runs)
         n_tok = min(wl.T, 32)
-        t0 = time.perf_counter()
-        oracle.forward(wl, inp, rows=list(range(n_tok)))
-        dt = time.perf_counter() - t0
-        cpu = {"value": n_tok / dt, "unit": "tokens/s", "cores": oracle.get_threads(), "kind": "oracle",
-               "sample": f"first {n_tok} tokens: full routing of all {wl.T} tokens plus the expert FFNs and "
-                         f"combine of the sampled ones ({dt:.1f} s)"}
+        dt, runs = 0.0, 0
+        while runs == 0 or (dt < 10.0 and runs < 8):
+            t0 = time.perf_counter()
+            oracle.forward(wl, inp, rows=list(range(n_tok)))
+            dt += time.perf_counter() - t0
+            runs += 1
+        cpu = {"value": n_tok * runs / dt, "unit": "tokens/s", "cores": oracle.get_threads(), "kind": "oracle",
+               "sample": f"first {n_tok} tokens, {runs} runs: full routing of all {wl.T} tokens plus the expert "
+                         f"FFNs and combine of the sampled ones ({dt:.1f} s)"}
 
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
