@@ -376,12 +376,13 @@ def main():
            "d2h_bytes_per_step": io_bytes}
 
     # kernels this library launched per step: gate logits + expert choice, 3 for the
-    # permutation, per FFN problem a schedule kernel + 2 (+ a row gather for the routed experts on the
-    # tensor-core routes, + 3 weight-decode passes on the decode-once route), combine
+    # permutation (one up to 1024 pairs), per FFN problem a schedule kernel + 2 (+ a row
+    # gather for the routed experts on the tensor-core routes, + 3 weight-decode passes on
+    # the decode-once route), combine
     def ffn_launches(r, routed):
         return 3 + (1 if routed and r in ("tc", "tc_dequant") else 0) + (3 if r == "tc_dequant" else 0)
 
-    per_step = 2 + 3 + ffn_launches(route, True) + 1
+    per_step = 2 + (1 if wl.P <= 1024 else 3) + ffn_launches(route, True) + 1
     if wl.has_shared:
         per_step += ffn_launches(gb.ffn_route(cfg, shared=True), False)
 

@@ -3,6 +3,7 @@
 // them into counts, offsets and per-block bases, and a scatter that ranks
 // pairs inside a block in pair order (warp match + warp-ordered running
 // counters), so the result is the stable order whatever the scheduling.
+// Up to 1024 pairs (decode) all three steps run in one CTA.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -103,9 +104,76 @@ perm_scatter_kernel(const int32_t* __restrict__ ids, int64_t P, int E, const int
     }
 }
 
+// P <= kPermBlock: histogram, scan and stable scatter in one CTA (one pair
+// per thread). Same order and outputs as the three kernels above with one
+// block: the block base of expert e is its offset.
+__global__ void __launch_bounds__(kPermBlock)
+perm_small_kernel(const int32_t* __restrict__ ids, int64_t P, int E, int32_t* __restrict__ counts,
+                  int32_t* __restrict__ offsets, int32_t* __restrict__ sorted_pair, int32_t* __restrict__ pair_pos) {
+    pdl_enter();
+    extern __shared__ int32_t s_run[];  // [E]: histogram, then running positions
+    __shared__ int32_t s_warp[kPermBlock / 32];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    for (int e = threadIdx.x; e < E; e += blockDim.x) s_run[e] = 0;
+    __syncthreads();
+    const int p = threadIdx.x;
+    const int id = p < P ? ids[p] : -1;
+    const bool valid = id >= 0 && id < E;  // out-of-range ids are dropped
+    if (valid) atomicAdd(&s_run[id], 1);
+    __syncthreads();
+    // exclusive scan of the counts over experts (thread e owns expert e; E <= 512)
+    const int cnt = threadIdx.x < E ? s_run[threadIdx.x] : 0;
+    int incl = cnt;
+#pragma unroll
+    for (int d = 1; d < 32; d <<= 1) {
+        int o = __shfl_up_sync(0xffffffffu, incl, d);
+        if (lane >= d) incl += o;
+    }
+    if (lane == 31) s_warp[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+        int w = s_warp[lane], wi = w;
+#pragma unroll
+        for (int d = 1; d < 32; d <<= 1) {
+            int o = __shfl_up_sync(0xffffffffu, wi, d);
+            if (lane >= d) wi += o;
+        }
+        s_warp[lane] = wi - w;  // exclusive warp prefix
+    }
+    __syncthreads();
+    const int excl = s_warp[warp] + incl - cnt;
+    if (threadIdx.x < E) {
+        counts[threadIdx.x] = cnt;
+        offsets[threadIdx.x] = excl;
+        if (threadIdx.x == E - 1) offsets[E] = excl + cnt;
+        s_run[threadIdx.x] = excl;
+    }
+    __syncthreads();
+    // stable scatter: warps take their places in pair order
+    const int e = valid ? id : -1 - lane;  // invalid lanes never match a real expert
+    const uint32_t peers = __match_any_sync(0xffffffffu, e);
+    const int rank = __popc(peers & ((1u << lane) - 1u));
+    int pos = 0;
+    for (int w = 0; w < kPermBlock / 32; ++w) {
+        if (warp == w && valid) {
+            pos = s_run[e] + rank;
+            __syncwarp(peers);
+            if (rank == 0) s_run[e] += __popc(peers);
+        }
+        __syncthreads();
+    }
+    if (valid) {
+        sorted_pair[pos] = p;
+        pair_pos[p] = pos;
+    }
+}
+
 cudaError_t launch_permute(const int32_t* topk_ids, int64_t P, int E, int32_t* counts, int32_t* offsets,
                            int32_t* sorted_pair, int32_t* pair_pos, int32_t* scratch, cudaStream_t stream) {
     const int nblk = permute_blocks(P);
+    if (nblk == 1)
+        return launch_k(perm_small_kernel, dim3(1), dim3(kPermBlock), E * sizeof(int32_t), stream, topk_ids, P, E,
+                        counts, offsets, sorted_pair, pair_pos);
     int32_t* block_hist = scratch;
     int32_t* block_base = scratch + (size_t)nblk * E;
     if (nblk > 0) {

@@ -111,10 +111,13 @@ def test_argument_errors_launch_nothing():
     assert e.value.status == gb.EINVAL
 
 
-@pytest.mark.parametrize("T,E,k,H", [(1100, 20, 3, 512), (1024, 16, 2, 256), (2049, 256, 8, 768)])
-def test_large_batch_routing_is_bit_exact(T, E, k, H):
-    # large batches take the tiled gate kernel: ragged token and expert tiles
-    wl = TINY.replace(T=T, E=E, top_k=k, H=H, act="bf16", wq="bf16", seed=T + E)
+@pytest.mark.parametrize("T,E,k,H,act", [(1100, 20, 3, 512, "bf16"), (1024, 16, 2, 256, "bf16"),
+                                         (2049, 256, 8, 768, "bf16"), (1100, 20, 3, 512, "f32"),
+                                         (1023, 20, 3, 512, "bf16"), (7, 256, 8, 768, "f32")])
+def test_batch_routing_is_bit_exact(T, E, k, H, act):
+    # bf16 batches from 1024 tokens take the tiled logits kernel, smaller ones
+    # and fp32 the per-warp one; ragged token and expert tiles
+    wl = TINY.replace(T=T, E=E, top_k=k, H=H, act=act, wq=act, seed=T + E)
     inp = synth.make_inputs(wl, with_experts=False)
     dev = to_device(wl, dict(inp, experts={}, shared=None))
     cfg = config(wl)
@@ -123,8 +126,8 @@ def test_large_batch_routing_is_bit_exact(T, E, k, H):
     w = torch.empty((T, k), dtype=torch.float32, device="cuda")
     gb.moe_route(cfg, dev["x"], dev["w_router"], None, None, ids, w, ws)
     torch.cuda.synchronize()
-    x32 = synth.bf16_bits_to_f32(inp["x"])
-    g32 = synth.bf16_bits_to_f32(inp["w_router"])
+    x32 = inp["x"] if act == "f32" else synth.bf16_bits_to_f32(inp["x"])
+    g32 = inp["w_router"] if act == "f32" else synth.bf16_bits_to_f32(inp["w_router"])
     ref_ids, ref_w = oracle.route(oracle.gate_logits(x32, g32), k)
     assert np.array_equal(ids.cpu().numpy(), ref_ids)
     np.testing.assert_allclose(w.cpu().numpy(), ref_w, rtol=2e-6, atol=1e-7)
