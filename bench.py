@@ -43,8 +43,8 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # line reports it times this run's active experts. Keyed by (workload, route);
 # absent (null) whenever the kernels changed since the counters were taken.
 # decode: stream_gateup + stream_down on T=8, E=32 (29 active experts):
-# 730.1 + 3.5 + 365.2 + 3.2 MB.
-TRAFFIC_PER_ACTIVE_EXPERT: dict = {("decode_bf16_T32_H4096_E128_k8_I1536", "stream"): 1101.981e6 / 29}
+# 730.0 + 3.2 + 365.2 + 3.2 MB.
+TRAFFIC_PER_ACTIVE_EXPERT: dict = {("decode_bf16_T32_H4096_E128_k8_I1536", "stream"): 1101.571e6 / 29}
 
 
 def peaks():
