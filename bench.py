@@ -189,6 +189,24 @@ def run_reference(args, wl, inp, rank):
             "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 
+def max_over_ranks(v: float, dist, device) -> float:
+    """The largest v over the process group (dist None: v): the slowest replica
+    sets the job's time."""
+    if dist is None:
+        return v
+    import torch
+
+    t = torch.tensor([v], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def replica_throughput(tokens_per_step: int, steps: int, world: int, seconds: float) -> float:
+    """Whole-job tokens/s of `world` independent replicas that each ran `steps`
+    steps of `tokens_per_step` tokens in `seconds` (the max over ranks)."""
+    return tokens_per_step * steps * world / seconds
+
+
 def workload_config(wl):
     return {"workload": wl.name, "T": wl.T, "H": wl.H, "I": wl.I, "E": wl.E, "top_k": wl.top_k,
             "scoring": wl.score, "activations": wl.act, "weights": wl.wq,
@@ -301,12 +319,8 @@ def main():
         end.record(stream)
         torch.cuda.synchronize()
     barrier()
-    ms = start.elapsed_time(end)
-    if dist is not None:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
-    value = wl.T * args.steps * world / (ms / 1e3)
+    ms = max_over_ranks(start.elapsed_time(end), dist, dev)
+    value = replica_throughput(wl.T, args.steps, world, ms / 1e3)
 
     # dominant kernel: the expert FFN, timed through its own entry point on the same stream
     P = wl.P
@@ -367,12 +381,10 @@ def main():
         stream.synchronize()
     e2e_s = time.perf_counter() - t0
     barrier()
-    if dist is not None:
-        t = torch.tensor([e2e_s], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_s = float(t.item())
+    e2e_s = max_over_ranks(e2e_s, dist, dev)
     io_bytes = wl.T * wl.H * x.element_size()
-    e2e = {"value": wl.T * args.steps * world / e2e_s, "unit": "tokens/s", "h2d_bytes_per_step": io_bytes,
+    e2e = {"value": replica_throughput(wl.T, args.steps, world, e2e_s), "unit": "tokens/s",
+           "h2d_bytes_per_step": io_bytes,
            "d2h_bytes_per_step": io_bytes}
 
     # kernels this library launched per step: gate logits + expert choice, 3 for the
