@@ -152,3 +152,17 @@ def test_streaming_column_groups_per_cta(T, E, k):
     got = act_np(out) if rows is None else act_np(out)[ref["rows"]]
     err = rel_err(got, ref["out"])
     assert err <= tol_for(wl), f"rel err {err:.3e}"
+
+
+# The largest expert count and top-k the configuration admits (E = 512,
+# top_k = 32), softmax and sigmoid with 32 groups, on every FFN route that
+# covers the activation dtype.
+@pytest.mark.parametrize("score,act,route", [("softmax", "f32", "stream"), ("softmax", "f32", "simt"),
+                                             ("softmax", "bf16", "tc"), ("sigmoid", "bf16", "stream")])
+def test_maximum_experts_and_top_k(score, act, route):
+    extra = dict(score="sigmoid", routed_scale=2.5, n_group=32, topk_group=4, select_bias_sigma=0.01) \
+        if score == "sigmoid" else {}
+    wl = TINY.replace(T=40, E=512, top_k=32, H=256, I=128, act=act, wq=act, seed=77, **extra)
+    assert gb.check_config(config(wl, route)) == gb.OK
+    ref = check(wl, route)
+    assert (ref["counts"] > 0).sum() > 200
