@@ -141,22 +141,25 @@ def load_workload(wid: int, overrides=()):
     return wl, inp
 
 
+def expert_bytes(wq: str, H: int, I: int) -> int:
+    """Bytes of one expert's gate, up and down matrices in storage format wq,
+    scales included."""
+    per = 3 * H * I
+    if wq == "bf16":
+        return per * 2
+    if wq == "f32":
+        return per * 4
+    if wq == "fp8_b128":  # e4m3 codes + one fp32 scale per 128x128 block
+        return per + 3 * (H // 128) * (I // 128) * 4
+    return per // 2 + 3 * (H * I // 128) * 2  # int4 nibbles + one bf16 scale per 128 along K
+
+
 def algorithmic_weight_bytes(wl, active: int) -> int:
     """Expert weight bytes one layer forward must read: every active expert's
     three matrices (+ scales), plus the shared expert."""
-    per = 3 * wl.H * wl.I
-    if wl.wq == "bf16":
-        b = per * 2
-    elif wl.wq == "f32":
-        b = per * 4
-    elif wl.wq == "fp8_b128":
-        b = per + 3 * (wl.H // 128) * (wl.I // 128) * 4
-    else:
-        b = per // 2 + 3 * (wl.H * wl.I // 128) * 2
-    total = active * b
+    total = active * expert_bytes(wl.wq, wl.H, wl.I)
     if wl.has_shared:
-        ps = 3 * wl.H * wl.I_shared
-        total += (ps + 3 * (wl.H // 128) * (wl.I_shared // 128) * 4) if wl.wq == "fp8_b128" else ps * 2
+        total += expert_bytes(wl.wq, wl.H, wl.I_shared)
     return total
 
 
