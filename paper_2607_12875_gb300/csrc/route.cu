@@ -32,6 +32,9 @@ gate_logits_kernel(const TA* __restrict__ x, const TA* __restrict__ wg, const fl
         for (int b = 0; b < kGateExpertsPerWarp; ++b) acc[a][b] = 0.0f;
 
     const int nchunk = H / 8;  // H % 256 == 0: every lane gets H/256 chunks
+    // two steps per iteration: their loads are in flight together (each
+    // accumulator still takes its chunks in increasing order)
+#pragma unroll 2
     for (int c = lane; c < nchunk; c += 32) {
         float xv[TB][8];
 #pragma unroll
