@@ -2,6 +2,7 @@
 #pragma once
 
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -124,6 +125,15 @@ __device__ __forceinline__ float e4m3_to_f32(uint32_t b) {
         mag = (float)em * 0.001953125f;  // m * 2^-9
     }
     return __uint_as_float(__float_as_uint(mag) | sign);
+}
+
+// two e4m3 values (low byte = first element) -> two fp32, through the
+// hardware e4m3x2 -> f16x2 conversion (every e4m3 value is exact in f16)
+__device__ __forceinline__ float2 e4m3x2_to_f32x2(uint32_t two_bytes) {
+    uint32_t h2;
+    asm("cvt.rn.f16x2.e4m3x2 %0, %1;" : "=r"(h2) : "h"((unsigned short)two_bytes));
+    __half2 h = *reinterpret_cast<__half2*>(&h2);
+    return __half22float2(h);
 }
 
 // signed 4-bit value of nibble n (two's complement)

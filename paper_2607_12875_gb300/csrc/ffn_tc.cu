@@ -267,14 +267,6 @@ __device__ __forceinline__ uint32_t sw128_off(int r, int c) { return (uint32_t)(
 __device__ __forceinline__ uint32_t sw64_off(int r, int c) { return (uint32_t)(r * 64 + ((c ^ ((r >> 1) & 3)) << 4)); }
 __device__ __forceinline__ uint32_t sw32_off(int r, int c) { return (uint32_t)(r * 32 + ((c ^ ((r >> 2) & 1)) << 4)); }
 
-// two e4m3 values (low byte = first element) -> two fp32
-__device__ __forceinline__ float2 e4m3x2_to_f32x2(uint32_t two_bytes) {
-    uint32_t h2;
-    asm("cvt.rn.f16x2.e4m3x2 %0, %1;" : "=r"(h2) : "h"((unsigned short)two_bytes));
-    __half2 h = *reinterpret_cast<__half2*>(&h2);
-    return __half22float2(h);
-}
-
 // 16 e4m3 weights (one 16-byte raw chunk) times the block scale -> 16 bf16 in two 16-byte chunks
 __device__ __forceinline__ void decode_fp8_16(const uint4 raw, float sc, uint4& o0, uint4& o1) {
     const uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};

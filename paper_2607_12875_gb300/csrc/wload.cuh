@@ -61,12 +61,11 @@ struct WFmt<GBMOE_FP8_E4M3_B128> {
     }
     __device__ static float scale_at(const void* row, int k) { return static_cast<const float*>(row)[k / 128]; }
     __device__ __forceinline__ static void decode8(const uint4 (&r)[NV], int sub, float sc, float (&w)[8]) {
-        uint32_t lo = sub ? r[0].z : r[0].x, hi = sub ? r[0].w : r[0].y;
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            w[i] = e4m3_to_f32((lo >> (8 * i)) & 0xffu) * sc;
-            w[4 + i] = e4m3_to_f32((hi >> (8 * i)) & 0xffu) * sc;
-        }
+        const uint32_t lo = sub ? r[0].z : r[0].x, hi = sub ? r[0].w : r[0].y;
+        const float2 a = e4m3x2_to_f32x2(lo & 0xffffu), b = e4m3x2_to_f32x2(lo >> 16);
+        const float2 c = e4m3x2_to_f32x2(hi & 0xffffu), d = e4m3x2_to_f32x2(hi >> 16);
+        w[0] = a.x * sc; w[1] = a.y * sc; w[2] = b.x * sc; w[3] = b.y * sc;
+        w[4] = c.x * sc; w[5] = c.y * sc; w[6] = d.x * sc; w[7] = d.y * sc;
     }
     __device__ static float elem(const void* w, const void* s, int64_t e, int N, int K, int n, int k) {
         uint32_t b = static_cast<const uint8_t*>(w)[((size_t)e * N + n) * K + k];
