@@ -210,6 +210,29 @@ def replica_throughput(tokens_per_step: int, steps: int, world: int, seconds: fl
     return tokens_per_step * steps * world / seconds
 
 
+def roofline_entry(alg_bytes: float, flops: float, ms: float, pk: dict, pk_kind: str, extra: dict) -> dict:
+    """The bench line's roofline object for one kernel call of `ms` milliseconds
+    that must move `alg_bytes` and do `flops`: bound by the slower of the bytes
+    over the HBM copy peak and the FLOPs over the bf16 dense peak. A
+    tensor-bound entry also gives the fraction of the sustained (power-capped)
+    bf16 peak, the denominator for kernels timed inside long runs."""
+    t_hbm = alg_bytes / (pk["hbm_gbs"] * 1e9)
+    t_tensor = flops / (pk["bf16_tflops"] * 1e12)
+    common = {**extra, "algorithmic_bytes": alg_bytes, "algorithmic_flops": flops, "ms_per_launch": ms,
+              "roofline_ms": max(t_hbm, t_tensor) * 1e3}
+    if t_hbm >= t_tensor:
+        achieved = alg_bytes / (ms / 1e3) / 1e9
+        return {"bound": "hbm", "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s",
+                "frac": achieved / pk["hbm_gbs"], "peak_kind": f"{pk_kind} HBM copy", **common}
+    achieved = flops / (ms / 1e3) / 1e12
+    entry = {"bound": "tensor", "achieved": achieved, "peak": pk["bf16_tflops"], "unit": "TFLOP/s",
+             "frac": achieved / pk["bf16_tflops"], "peak_kind": f"{pk_kind} bf16 dense burst"}
+    sustained = pk.get("bf16_tflops_sustained")
+    if sustained:
+        entry.update(peak_sustained=sustained, frac_sustained=achieved / sustained)
+    return {**entry, **common}
+
+
 def workload_config(wl):
     return {"workload": wl.name, "T": wl.T, "H": wl.H, "I": wl.I, "E": wl.E, "top_k": wl.top_k,
             "scoring": wl.score, "activations": wl.act, "weights": wl.wq,
@@ -351,25 +374,14 @@ def main():
     # HBM bandwidth and its FLOPs over the bf16 tensor peak
     routed_bytes = algorithmic_weight_bytes(wl.replace(has_shared=False), active)
     flops = 6.0 * wl.P * wl.H * wl.I
-    t_hbm = routed_bytes / (pk["hbm_gbs"] * 1e9)
-    t_tensor = flops / (pk["bf16_tflops"] * 1e12)
     kernel = {"stream": "moe_grouped_ffn, weight-streaming route (gate/up + down)",
               "tc": "moe_grouped_ffn, tcgen05 route (row gather + gate/up GEMM with SwiGLU + down GEMM)",
               "tc_dequant": "moe_grouped_ffn, tcgen05 decode-once route (3 weight-decode passes + row gather + "
                             "gate/up GEMM with SwiGLU + down GEMM)",
               "simt": "moe_grouped_ffn, CUDA-core route"}[route]
     tpe = TRAFFIC_PER_ACTIVE_EXPERT.get((wl.name, route))
-    common = {"traffic": None if tpe is None else tpe * active, "kernel": kernel, "algorithmic_bytes": routed_bytes,
-              "algorithmic_flops": flops, "active_experts": active, "ms_per_launch": ffn_ms,
-              "roofline_ms": max(t_hbm, t_tensor) * 1e3}
-    if t_hbm >= t_tensor:
-        achieved = routed_bytes / (ffn_ms / 1e3) / 1e9
-        roofline = {"bound": "hbm", "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s",
-                    "frac": achieved / pk["hbm_gbs"], "peak_kind": f"{pk_kind} HBM copy", **common}
-    else:
-        achieved = flops / (ffn_ms / 1e3) / 1e12
-        roofline = {"bound": "tensor", "achieved": achieved, "peak": pk["bf16_tflops"], "unit": "TFLOP/s",
-                    "frac": achieved / pk["bf16_tflops"], "peak_kind": f"{pk_kind} bf16 dense burst", **common}
+    extra = {"traffic": None if tpe is None else tpe * active, "kernel": kernel, "active_experts": active}
+    roofline = roofline_entry(routed_bytes, flops, ffn_ms, pk, pk_kind, extra)
 
     # end to end through the public host-buffer entry point
     x_host = x.cpu().pin_memory()
