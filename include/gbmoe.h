@@ -150,11 +150,12 @@ int moe_route(const gbmoe_config* cfg, const void* x, const void* w_router, cons
 
 /*
  * Fused MoE, grouping step: stable counting sort of the P pairs by expert.
- * topk_ids [T, k] int32 (each in [0, E); out-of-range ids are not checked on
- * the device and give undefined grouping). Writes counts [E], offsets [E+1]
+ * topk_ids [T, k] int32, each in [0, E). Writes counts [E], offsets [E+1]
  * (exclusive prefix sum, offsets[E] = P), sorted_pair [P] (pairs ordered by
  * expert, then by pair index) and pair_pos [P] (inverse: position of pair p),
- * all int32. Bit-exact and deterministic.
+ * all int32. Bit-exact and deterministic. A pair whose id is out of range is
+ * dropped: not counted, no slot (offsets[E] is then below P, and the tail of
+ * sorted_pair and that pair's pair_pos entry are left unwritten).
  */
 int moe_permute(const gbmoe_config* cfg, const int32_t* topk_ids, int32_t* counts, int32_t* offsets,
                 int32_t* sorted_pair, int32_t* pair_pos, void* workspace, size_t workspace_bytes,
