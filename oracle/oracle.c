@@ -119,7 +119,8 @@ int oracle_gate_logits(int64_t T, int64_t H, int64_t E, const float* x, const fl
  * Pinned fp32 exponential, used where an exponential decides the expert
  * choice (sigmoid scores plus a selection bias). Written from the
  * mathematics, not from any library:
- *   clamp x to [-86, 88] so that the result stays a normal number;
+ *   a NaN is returned as it is; otherwise clamp x to [-86, 88] so that the
+ *   result stays a normal number;
  *   n = rint(x * log2(e));  r = (x - n*ln2_hi) - n*ln2_lo  (Cody and Waite,
  *   "Software Manual for the Elementary Functions", 1980: ln2_hi keeps the
  *   leading 16 bits of ln 2 so that n*ln2_hi is exact);
@@ -137,6 +138,7 @@ float oracle_pexp(float x) {
     static const uint32_t inv_fact[9] = {              /* fp32(1/i!), i = 0..8   */
         0x3f800000u, 0x3f800000u, 0x3f000000u, 0x3e2aaaabu, 0x3d2aaaabu,
         0x3c088889u, 0x3ab60b61u, 0x39500d01u, 0x37d00d01u};
+    if (isnan(x)) return x; /* NaN in, NaN out, as for exp */
     if (x < -86.0f) x = -86.0f;
     if (x > 88.0f) x = 88.0f;
     float t = x * log2e;
@@ -165,6 +167,12 @@ typedef struct {
     int32_t n_group, topk_group;
     float routed_scale;
 } oracle_route_cfg;
+
+/* Key a score takes in the expert choice. Reading (the paper is silent on
+ * non-finite scores): a NaN counts as -infinity, so that every comparison
+ * below is a total order and the choice stays defined; ties, as always, go
+ * to the lower index. */
+static float choice_key(float v) { return isnan(v) ? -INFINITY : v; }
 
 /* Index of the largest key among those with allowed[e] != 0; the lowest index
  * wins a tie (the scan is ascending and only a strictly larger key replaces). */
@@ -221,11 +229,11 @@ int oracle_route(const oracle_route_cfg* c, const float* logits, const float* se
         int32_t* id = ids + t * k;
         double* wt = w + t * k;
         if (c->score == 0) {
-            for (int e = 0; e < E; ++e) { key[e] = l[e]; allowed[e] = 1; }
+            for (int e = 0; e < E; ++e) { key[e] = choice_key(l[e]); allowed[e] = 1; }
         } else {
             for (int e = 0; e < E; ++e) {
                 s[e] = oracle_sigmoid(l[e]);
-                key[e] = select_bias ? s[e] + select_bias[e] : s[e];
+                key[e] = choice_key(select_bias ? s[e] + select_bias[e] : s[e]);
                 allowed[e] = 1;
             }
             if (G > 1) {
@@ -237,7 +245,7 @@ int oracle_route(const oracle_route_cfg* c, const float* logits, const float* se
                         if (a < 0 || key[e] > key[a]) { b = a; a = e; }
                         else if (b < 0 || key[e] > key[b]) b = e;
                     }
-                    gscore[g] = key[a] + key[b];
+                    gscore[g] = choice_key(key[a] + key[b]);
                     gallowed[g] = 1;
                 }
                 unsigned char* kept = (unsigned char*)calloc(G, 1);

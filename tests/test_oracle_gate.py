@@ -79,3 +79,11 @@ def test_sigmoid_against_math():
     ulp = np.spacing(ref.astype(np.float32)).astype(np.float64)
     assert np.max(np.abs(got - ref) / ulp) <= 4.0
     assert oracle.sigmoid(np.array([0.0], np.float32))[0] == 0.5
+
+
+def test_pexp_and_sigmoid_propagate_nan():
+    """NaN in, NaN out, as for exp (the clamp does not turn NaN into a number)."""
+    got = oracle.pexp(np.array([np.nan, -np.nan], np.float32))
+    assert np.isnan(got).all()
+    assert np.isnan(oracle.sigmoid(np.array([np.nan], np.float32))).all()
+    assert oracle.pexp(np.array([np.inf], np.float32))[0] == oracle.pexp(np.array([88.0], np.float32))[0]

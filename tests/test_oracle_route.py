@@ -2,6 +2,7 @@
 scipy's softmax, the hand cases in tests/golden/hand_cases.json and the
 defining properties of group-limited selection."""
 import json
+import math
 import os
 
 import numpy as np
@@ -115,3 +116,40 @@ def test_route_rejects_invalid_configurations():
         oracle.route(l, 2, "sigmoid", True, 3, 1)
     with pytest.raises(ValueError):
         oracle.route(l, 5, "sigmoid", True, 4, 2)  # only 4 experts in 2 groups of 2
+
+
+def _nan_last(v):
+    """Sort key of the choice's reading for non-finite scores: NaN counts as -inf."""
+    v = float(v)
+    return -math.inf if math.isnan(v) else v
+
+
+def test_nan_scores_rank_as_minus_infinity():
+    """Non-finite logits still give valid ids: a NaN key counts as -inf, ties
+    (among NaN and -inf keys too) go to the lower index."""
+    rng = np.random.default_rng(11)
+    E, k = 16, 6
+    logits = rng.integers(-2, 3, size=(200, E)).astype(np.float32)
+    logits[rng.random((200, E)) < 0.3] = np.nan
+    logits[rng.random((200, E)) < 0.1] = -np.inf
+    logits[5] = np.nan  # a token whose every logit is NaN
+    ids, _ = oracle.route(logits, k)
+    for t in range(200):
+        assert list(ids[t]) == sorted(range(E), key=lambda e: (-_nan_last(logits[t, e]), e))[:k]
+    assert list(ids[5]) == list(range(k))
+    # sigmoid, group-limited, NaN selection biases
+    bias = np.zeros(E, np.float32)
+    bias[[1, 9]] = np.nan
+    ids2, _ = oracle.route(logits, 4, "sigmoid", True, 4, 2, 1.0, bias)
+    assert ((ids2 >= 0) & (ids2 < E)).all()
+    q = (oracle.sigmoid(logits) + bias[None, :]).astype(np.float32)
+    for t in range(200):
+        key = [_nan_last(v) for v in q[t]]
+        gscore = []
+        for g in range(4):
+            top2 = sorted(key[4 * g:4 * g + 4], reverse=True)[:2]
+            s = np.float32(top2[0]) + np.float32(top2[1])
+            gscore.append(_nan_last(s))
+        kept = sorted(range(4), key=lambda g: (-gscore[g], g))[:2]
+        cand = [e for e in range(E) if e // 4 in kept]
+        assert list(ids2[t]) == sorted(cand, key=lambda e: (-key[e], e))[:4]
