@@ -154,8 +154,11 @@ int moe_route(const gbmoe_config* cfg, const void* x, const void* w_router, cons
  * (exclusive prefix sum, offsets[E] = P), sorted_pair [P] (pairs ordered by
  * expert, then by pair index) and pair_pos [P] (inverse: position of pair p),
  * all int32. Bit-exact and deterministic. A pair whose id is out of range is
- * dropped: not counted, no slot (offsets[E] is then below P, and the tail of
- * sorted_pair and that pair's pair_pos entry are left unwritten).
+ * dropped: it is not counted and gets no slot; its pair_pos entry is -1,
+ * offsets[E] is then below P, and sorted_pair[offsets[E] .. P-1] hold -1.
+ * moe_grouped_ffn and moe_combine accept these outputs as they are: the FFN
+ * computes only the counted rows, and a dropped pair adds nothing to its
+ * token's output.
  */
 int moe_permute(const gbmoe_config* cfg, const int32_t* topk_ids, int32_t* counts, int32_t* offsets,
                 int32_t* sorted_pair, int32_t* pair_pos, void* workspace, size_t workspace_bytes,
@@ -186,7 +189,8 @@ int moe_shared_ffn(const gbmoe_config* cfg, const void* x, const gbmoe_expert_we
  *   out[t] = sum_{j=0..k-1} topk_w[t,j] * y_pairs[pair_pos[t*k + j]]
  *            (+ y_shared[t] if y_shared is not NULL),
  * summed in fp32 in that order and rounded once to act_dtype. A gather per
- * token: no atomics, deterministic. y_pairs [P, H], y_shared [T, H] or NULL,
+ * token: no atomics, deterministic. Slots with a negative pair_pos (pairs
+ * moe_permute dropped) are skipped. y_pairs [P, H], y_shared [T, H] or NULL,
  * out [T, H], all act_dtype; topk_w [T, k] fp32; pair_pos [P] int32.
  */
 int moe_combine(const gbmoe_config* cfg, const void* y_pairs, const float* topk_w, const int32_t* pair_pos,
@@ -220,6 +224,11 @@ int moe_forward_hostio(const gbmoe_config* cfg, const void* x_host, const void* 
  * Reads (and clears) the device error word that bounded device-side waits
  * set in `workspace`, after synchronising `stream`. *status receives GBMOE_OK
  * or GBMOE_EDEVICE_TIMEOUT. This is the only call that synchronises.
+ * The waits are those of the tensor-core FFN kernels (GBMOE_FFN_TC and
+ * _TC_DEQUANT): each gives up after 2 s, stops issuing work, lets the copies
+ * and MMAs it issued finish, and sets the word; the call's outputs are then
+ * incomplete. For tests of this path the environment variable
+ * GBMOE_TC_WAIT_LIMIT_NS (read at every call) lowers the limit, in ns.
  */
 int moe_device_status(void* workspace, void* stream, int32_t* status);
 

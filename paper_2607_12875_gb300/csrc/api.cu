@@ -14,7 +14,6 @@ using namespace gbmoe;
 namespace {
 
 constexpr size_t kAlign = 256;
-constexpr size_t kSmemBudget = 227 * 1024;  // per-CTA shared memory on sm_103a
 
 size_t align_up(size_t v) { return (v + kAlign - 1) & ~(kAlign - 1); }
 
@@ -51,7 +50,7 @@ int check_cfg(const gbmoe_config* c) {
     return GBMOE_OK;
 }
 
-bool stream_fits(int act_dtype, int H, int I) { return stream_smem_bytes(act_dtype, H, I) <= kSmemBudget; }
+bool stream_fits(int act_dtype, int H, int I) { return stream_smem_bytes(act_dtype, H, I) <= stream_smem_budget(); }
 
 // Kernel route for an FFN problem with n_rows rows over E experts.
 int pick_route(const gbmoe_config* c, int64_t n_rows, int E, int I) {
@@ -147,22 +146,33 @@ RouteParams route_params(const gbmoe_config* c) {
     return rp;
 }
 
-int run_ffn(const gbmoe_config* c, FfnProblem& p, int route, cudaStream_t stream) {
-    cudaError_t err;
+// GBMOE_OK when an FFN problem of intermediate size I can run on `route`,
+// checked on the host so that a call fails before it enqueues anything.
+int route_launchable(const gbmoe_config* c, int route, int I) {
     switch (route) {
-        case GBMOE_FFN_STREAM:
-            if (!stream_fits(p.act_dtype, p.H, p.I)) return GBMOE_EUNSUPPORTED;
-            err = launch_ffn_stream(p, stream);
-            break;
-        case GBMOE_FFN_SIMT: err = launch_ffn_simt(p, stream); break;
+        case GBMOE_FFN_STREAM: return stream_fits(c->act_dtype, c->H, I) ? GBMOE_OK : GBMOE_EUNSUPPORTED;
+        case GBMOE_FFN_SIMT: return GBMOE_OK;
         case GBMOE_FFN_TC:
-        case GBMOE_FFN_TC_DEQUANT:
-            if (!ffn_tc_supported(p)) return GBMOE_EUNSUPPORTED;
-            err = launch_ffn_tc(p, stream);
-            break;
+        case GBMOE_FFN_TC_DEQUANT: {
+            FfnProblem probe{};
+            probe.act_dtype = c->act_dtype;
+            probe.w_dtype = c->w_dtype;
+            probe.H = c->H;
+            probe.I = I;
+            return ffn_tc_supported(probe) ? GBMOE_OK : GBMOE_EUNSUPPORTED;
+        }
         default: return GBMOE_EINVAL;
     }
-    (void)c;
+}
+
+int run_ffn(const gbmoe_config* c, FfnProblem& p, int route, cudaStream_t stream) {
+    if (int s = route_launchable(c, route, p.I)) return s;
+    cudaError_t err;
+    switch (route) {
+        case GBMOE_FFN_STREAM: err = launch_ffn_stream(p, stream); break;
+        case GBMOE_FFN_SIMT: err = launch_ffn_simt(p, stream); break;
+        default: err = launch_ffn_tc(p, stream); break;  // GBMOE_FFN_TC, GBMOE_FFN_TC_DEQUANT
+    }
     return cuda_status(err);
 }
 
@@ -317,15 +327,13 @@ int moe_forward(const gbmoe_config* cfg, const void* x, const void* w_router, co
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     const Layout L = layout(cfg);
     const int64_t P = (int64_t)cfg->T * cfg->top_k;
-    // every route must be launchable before anything is enqueued
+    // every route must be launchable before anything is enqueued: the routed
+    // problem with I, the shared one with I_shared
     const int r_routed = pick_route(cfg, P, cfg->E, cfg->I);
+    if ((s = route_launchable(cfg, r_routed, cfg->I))) return s;
     const int r_shared = cfg->has_shared ? pick_route(cfg, cfg->T, 1, cfg->I_shared) : GBMOE_FFN_SIMT;
-    for (int r : {r_routed, r_shared}) {
-        if (r == GBMOE_FFN_STREAM && !stream_fits(cfg->act_dtype, cfg->H, r == r_routed ? cfg->I : cfg->I_shared))
-            return GBMOE_EUNSUPPORTED;
-    }
+    if (cfg->has_shared && (s = route_launchable(cfg, r_shared, cfg->I_shared))) return s;
     if (cudaMemsetAsync(at<int32_t>(ws, L.err), 0, 4, st) != cudaSuccess) return GBMOE_ECUDA;
-    if (cfg->T == 0) return GBMOE_OK;
     int32_t* ids = at<int32_t>(ws, L.ids);
     float* w = at<float>(ws, L.w);
     int32_t* counts = at<int32_t>(ws, L.counts);

@@ -1,6 +1,8 @@
 // Weight Sum: out[t] = sum_j w[t,j] * y_pairs[pair_pos[t*k + j]] (+ y_shared[t]).
 // One block per token gathers its k expert rows; fp32 sums in slot order,
 // rounded once. No atomics, so the result does not depend on scheduling.
+// A slot whose pair_pos is negative (a pair the permutation dropped) is
+// skipped.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -22,6 +24,7 @@ combine_kernel(const TA* __restrict__ y, const float* __restrict__ w, const int3
     for (int c = threadIdx.x; c < H / 8; c += blockDim.x) {
         float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
         for (int j = 0; j < k; ++j) {
+            if (s_pos[j] < 0) continue;  // a dropped pair contributes nothing
             float v[8];
             Vec8<TA>::load(y + (size_t)s_pos[j] * H + 8 * c, v);
             const float wj = s_w[j];

@@ -6,6 +6,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
 #include "../../include/gbmoe.h"
 
 namespace gbmoe {
@@ -42,6 +44,44 @@ cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t sme
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
+}
+
+// ------------------------------------------------- per-device host state
+
+constexpr int kMaxDevices = 64;
+
+// Runs a setup step (a cudaFuncSetAttribute, say) once per device: run(f)
+// calls f only while it has not yet succeeded on the current device. Two
+// threads racing on the first call may both run f, which is harmless for the
+// idempotent steps it is used for.
+struct DeviceOnce {
+    std::atomic<uint64_t> done{0};
+    template <typename F>
+    cudaError_t run(F&& f) {
+        int dev = 0;
+        if (cudaError_t e = cudaGetDevice(&dev); e != cudaSuccess) return e;
+        const uint64_t bit = dev >= 0 && dev < kMaxDevices ? 1ull << dev : 0;
+        if (bit && (done.load(std::memory_order_acquire) & bit)) return cudaSuccess;
+        const cudaError_t e = f();
+        if (e == cudaSuccess && bit) done.fetch_or(bit, std::memory_order_release);
+        return e;
+    }
+};
+
+// Number of SMs of the current device, queried once per device.
+inline int sm_count() {
+    static std::atomic<int> cache[kMaxDevices];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 1;
+    const bool cacheable = dev >= 0 && dev < kMaxDevices;
+    if (cacheable) {
+        if (const int n = cache[dev].load(std::memory_order_relaxed); n > 0) return n;
+    }
+    int n = 0;
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) return 1;
+    if (cacheable) cache[dev].store(n, std::memory_order_relaxed);
+    return n;
 }
 
 // ------------------------------------------------------------ bf16 helpers

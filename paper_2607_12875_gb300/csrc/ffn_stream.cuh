@@ -223,10 +223,7 @@ stream_down_kernel(FfnProblem p, int gpc) {
 // kMinWaves waves of CTAs (fewer, longer CTAs stage the rows less often;
 // too few CTAs leave SMs idle). groups is a multiple of 8.
 inline int groups_per_cta(int max_active, int groups) {
-    int sms = 0, dev = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    const int64_t slots = (int64_t)(sms > 0 ? sms : 1) * 2;  // resident CTAs (two per SM)
+    const int64_t slots = (int64_t)sm_count() * 2;  // resident CTAs (two per SM)
     int gpc = kMaxGroupsPerCta;
     while (gpc > 1 && (int64_t)max_active * (groups / gpc) < kMinWaves * slots) gpc /= 2;
     return gpc;
@@ -239,9 +236,15 @@ static cudaError_t launch_stream_t(const FfnProblem& p, cudaStream_t stream) {
     const size_t smem1 = (size_t)kNT * p.H * sizeof(TA);
     const size_t smem2 = (size_t)kNT * p.I * sizeof(TA);
     cudaError_t err;
-    err = cudaFuncSetAttribute(stream_gateup_kernel<TA, WQ>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem1);
-    if (err != cudaSuccess) return err;
-    err = cudaFuncSetAttribute(stream_down_kernel<TA, WQ>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem2);
+    // the largest dynamic shared memory any problem may ask for, set once per device
+    static DeviceOnce smem_set;
+    err = smem_set.run([] {
+        const int most = (int)stream_smem_budget();
+        cudaError_t e = cudaFuncSetAttribute(stream_gateup_kernel<TA, WQ>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, most);
+        if (e != cudaSuccess) return e;
+        return cudaFuncSetAttribute(stream_down_kernel<TA, WQ>, cudaFuncAttributeMaxDynamicSharedMemorySize, most);
+    });
     if (err != cudaSuccess) return err;
     const int groups1 = p.I / (2 * kStreamWarps), groups2 = p.H / (4 * kStreamWarps);
     const int gpc1 = groups_per_cta(max_active, groups1), gpc2 = groups_per_cta(max_active, groups2);

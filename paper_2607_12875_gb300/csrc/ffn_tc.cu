@@ -30,11 +30,13 @@
 // weight tile again, the caller's workspace instead receives one bf16 copy
 // of the active experts' weights (dequant_weights_kernel, same decode) and
 // the bf16 GEMM runs on it.
-// Every mbarrier wait is bounded (about two seconds); on expiry the CTA sets
-// the device error word, stops issuing work, drains what it issued and
+// Every mbarrier wait is bounded (two seconds by default); on expiry the CTA
+// sets the device error word, stops issuing work, drains what it issued and
 // frees its TMEM.
 #include <cuda.h>
 #include <cuda_fp16.h>
+
+#include <cstdlib>
 
 #include "common.cuh"
 #include "ffn_sched.h"
@@ -48,7 +50,7 @@ constexpr int A_BYTES = BM * BK * 2;
 constexpr int B_BYTES = BN * BK * 2;
 constexpr int TMEM_COLS = 512;
 constexpr int CONVERT_WARPS = 8;  // one thread per B row (BN = 256)
-constexpr unsigned long long kWaitLimitNs = 2000000000ull;
+constexpr unsigned long long kWaitLimitNs = 2000000000ull;  // default limit of a pipeline wait, and of every drain wait
 constexpr int kFp8PrefetchAhead = 4;  // k-blocks the fp8 producer prefetches into L2 ahead of its loads
 
 // Per weight format: bytes of the raw B tile TMA brings in (0 = B is loaded
@@ -96,6 +98,7 @@ struct Params {
     int32_t* err;
     const void* scale0;  // scales of the B rows in the first / second half of the tile
     const void* scale1;
+    uint64_t wait_limit_ns;  // limit of each pipeline wait (kWaitLimitNs unless a test shortens it)
 };
 
 // ------------------------------------------------------------ PTX wrappers
@@ -136,19 +139,39 @@ __device__ __forceinline__ uint64_t global_ns() {
 }
 
 // Bounded wait for the phase of `bar` with the given parity. Returns false
-// (after flagging the CTA and the device error word) when the limit expires
-// or another role of this CTA has already given up.
-__device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int32_t* err) {
+// (after flagging the CTA and the device error word) when `limit_ns` expires
+// or another role of this CTA has already given up. The clock is read after
+// every failed poll, so a wait longer than the limit always gives up.
+__device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int32_t* err,
+                                       uint64_t limit_ns) {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = global_ns();
-    for (uint32_t i = 1;; ++i) {
+    for (;;) {
         if (mbar_try_wait(bar, parity)) return true;
         if (*abort_flag) return false;
-        if ((i & 255u) == 0 && global_ns() - t0 > kWaitLimitNs) {
+        if (global_ns() - t0 > limit_ns) {
             *abort_flag = 1;
             set_error(err, kErrTimeout);
             return false;
         }
+    }
+}
+
+// The same wait by every lane of a warp, with one outcome for the whole warp:
+// if any lane gave up, all of them return false together, so no lane goes on
+// to a warp-synchronous step (__syncwarp, tcgen05.ld) its neighbours skip.
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int32_t* err,
+                                          uint64_t limit_ns) {
+    const bool ok = mbar_wait(bar, parity, abort_flag, err, limit_ns);
+    return __all_sync(0xffffffffu, ok);
+}
+
+// Waits (at most kWaitLimitNs) for a phase that work this thread issued will
+// complete; used at exit so that no copy or MMA is still in flight when the
+// CTA releases its shared memory and TMEM.
+__device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
+    const uint64_t t0 = global_ns();
+    while (!mbar_try_wait(bar, parity) && global_ns() - t0 < kWaitLimitNs) {
     }
 }
 
@@ -401,7 +424,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
                     tma_prefetch_2d(&tm_b0, xp, b0);
                     tma_prefetch_2d(&tm_b1, xp, b1);
                 }
-                if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, p.err)) { ok = false; break; }
+                if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, p.err, p.wait_limit_ns)) { ok = false; break; }
                 inflight &= ~(1u << stage);
                 mbar_expect_tx(&full[stage], A_BYTES + (RAW ? RAW : B_BYTES));
                 tma_load_2d(sA + stage * A_BYTES, &tm_a, kb * BK, (int)wk.row0, &full[stage]);
@@ -419,15 +442,11 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
                 if (++stage == STAGES) { stage = 0; phase ^= 1; }
             }
         }
-        if (!ok) {
-            // let the copies already issued land before the CTA leaves
-            for (int s = 0; s < STAGES; ++s) {
-                if (!((inflight >> s) & 1u)) continue;
-                const uint64_t t0 = global_ns();
-                while (!mbar_try_wait(&full[s], (inflight_par >> s) & 1u) && global_ns() - t0 < kWaitLimitNs) {
-                }
-            }
-        }
+        // let every copy issued land before the CTA leaves: after a normal run
+        // these phases have completed already; after an abort (here or in
+        // another role) the last loads may still be in flight
+        for (int s = 0; s < STAGES; ++s)
+            if ((inflight >> s) & 1u) drain_wait(&full[s], (inflight_par >> s) & 1u);
     } else if (warp == 1 && lane == 0) {
         // ------------------------------------------------------ MMA issuer
         int stage = 0;
@@ -437,12 +456,12 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
         bool ok = true;
         bool issued = false;
         for (int w = blockIdx.x; w < total && ok; w += gridDim.x) {
-            if (!mbar_wait(&tempty[acc], acc_phase ^ 1, abort_flag, p.err)) { ok = false; break; }
+            if (!mbar_wait(&tempty[acc], acc_phase ^ 1, abort_flag, p.err, p.wait_limit_ns)) { ok = false; break; }
             tc_fence_after();
             const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
             for (int kb = 0; kb < nkb; ++kb) {
-                if (!mbar_wait(&full[stage], phase, abort_flag, p.err)) { ok = false; break; }
-                if (RAW && !mbar_wait(&conv[stage], phase, abort_flag, p.err)) { ok = false; break; }
+                if (!mbar_wait(&full[stage], phase, abort_flag, p.err, p.wait_limit_ns)) { ok = false; break; }
+                if (RAW && !mbar_wait(&conv[stage], phase, abort_flag, p.err, p.wait_limit_ns)) { ok = false; break; }
                 tc_fence_after();
                 const uint64_t da = sw128_desc(smem_u32(sA + stage * A_BYTES));
                 const uint64_t db = sw128_desc(smem_u32(sB + stage * B_BYTES));
@@ -457,12 +476,12 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
             mma_commit(&tfull[acc]);
             if (++acc == 2) { acc = 0; acc_phase ^= 1; }
         }
-        if (!ok && issued) {
-            // wait for the MMAs already issued before TMEM is released
+        if (issued) {
+            // every MMA issued has finished before TMEM is released (after a
+            // normal run the epilogue has seen them all; after an abort in
+            // another role this issuer may have run up to two tiles ahead)
             mma_commit(drain);
-            const uint64_t t0 = global_ns();
-            while (!mbar_try_wait(drain, 0) && global_ns() - t0 < kWaitLimitNs) {
-            }
+            drain_wait(drain, 0);
         }
     } else if (warp >= 2 && warp < 6) {
         // -------------------------------------------------------- epilogue
@@ -474,7 +493,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
         uint32_t acc_phase = 0;
         for (int w = blockIdx.x; w < total; w += gridDim.x) {
             const Work wk = decode_work(p, w);
-            if (!mbar_wait(&tfull[acc], acc_phase, abort_flag, p.err)) break;
+            if (!warp_wait(&tfull[acc], acc_phase, abort_flag, p.err, p.wait_limit_ns)) break;
             tc_fence_after();
             const uint32_t t_row = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
             const bool valid = r < wk.rows;
@@ -541,7 +560,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
                     sc0 = sc1; sc1 = sc2; sc2 = sc3;
                     sc3 = scale_of(kb / 2 + 3);
                 }
-                if (!mbar_wait(&full[stage], phase, abort_flag, p.err)) { ok = false; break; }
+                if (!warp_wait(&full[stage], phase, abort_flag, p.err, p.wait_limit_ns)) { ok = false; break; }
                 const uint8_t* raw = sR + stage * RAW;
                 uint8_t* dstB = sB + stage * B_BYTES;
                 if (WQ == GBMOE_FP8_E4M3_B128) {
@@ -591,8 +610,8 @@ gather_rows_kernel(const uint4* __restrict__ x, const int32_t* __restrict__ sort
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
         const int64_t r = i / vec_per_row;
         const int c = (int)(i - r * vec_per_row);
-        const int64_t src = sorted_pair[r] / pair_div;
-        out[i] = x[src * vec_per_row + c];
+        const int32_t pr = sorted_pair[r];  // -1 past the last kept pair: a zero row
+        out[i] = pr >= 0 ? x[(int64_t)(pr / pair_div) * vec_per_row + c] : make_uint4(0, 0, 0, 0);
     }
 }
 
@@ -661,18 +680,18 @@ using EncodeTiled = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, 
                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
+// cuTensorMapEncodeTiled from the driver, looked up once per process (a
+// function-local static: its initialisation is thread-safe), or null.
 static EncodeTiled encode_fn() {
-    static EncodeTiled fn = nullptr;
-    static bool tried = false;
-    if (!tried) {
-        tried = true;
+    static const EncodeTiled fn = [] {
         void* ptr = nullptr;
         cudaDriverEntryPointQueryResult q;
         if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
                 cudaSuccess &&
             q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<EncodeTiled>(ptr);
-    }
+            return reinterpret_cast<EncodeTiled>(ptr);
+        return static_cast<EncodeTiled>(nullptr);
+    }();
     return fn;
 }
 
@@ -711,20 +730,16 @@ static bool map_weights(CUtensorMap* m, int wq, const void* base, int64_t rows, 
     }
 }
 
-static int num_sms() {
-    int dev = 0, n = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-    return n > 0 ? n : 1;
-}
-
 template <int WQ>
 static cudaError_t launch_gemm_t(const CUtensorMap& a, const CUtensorMap& b0, const CUtensorMap& b1,
                                  const CUtensorMap& out, const Params& prm, int64_t max_work, cudaStream_t stream) {
-    cudaError_t e = cudaFuncSetAttribute(tc_gemm_kernel<WQ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         Layout<WQ>::SMEM_BYTES);
+    static DeviceOnce smem_set;
+    cudaError_t e = smem_set.run([] {
+        return cudaFuncSetAttribute(tc_gemm_kernel<WQ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    Layout<WQ>::SMEM_BYTES);
+    });
     if (e != cudaSuccess) return e;
-    const int grid = (int)min64(num_sms(), max_work);
+    const int grid = (int)min64(sm_count(), max_work);
     if (grid <= 0) return cudaSuccess;
     if (const cudaError_t le = launch_k(tc_gemm_kernel<WQ>, dim3(grid), dim3(Fmt<WQ>::THREADS),
             Layout<WQ>::SMEM_BYTES, stream, a, b0, b1, out, prm); le != cudaSuccess)
@@ -777,6 +792,18 @@ static cudaError_t dequant_all(const FfnProblem& p, FfnProblem& q, cudaStream_t 
     return cudaSuccess;
 }
 
+// Limit of each pipeline wait of the GEMM kernels: kWaitLimitNs, or a shorter
+// one from GBMOE_TC_WAIT_LIMIT_NS (read at every call; for tests that make a
+// wait run out and check that the device error word reports it).
+static uint64_t wait_limit_ns() {
+    const char* v = std::getenv("GBMOE_TC_WAIT_LIMIT_NS");
+    if (!v || !*v) return tc::kWaitLimitNs;
+    char* end = nullptr;
+    const unsigned long long n = std::strtoull(v, &end, 10);
+    if (end == v || *end != '\0') return tc::kWaitLimitNs;
+    return n < tc::kWaitLimitNs ? n : tc::kWaitLimitNs;
+}
+
 cudaError_t launch_ffn_tc(const FfnProblem& pin, cudaStream_t stream) {
     using namespace tc;
     if (pin.n_rows == 0) return cudaSuccess;
@@ -813,6 +840,7 @@ cudaError_t launch_ffn_tc(const FfnProblem& pin, cudaStream_t stream) {
     g.counts = p.counts; g.offsets = p.offsets; g.sched = p.sched; g.E = p.E; g.n_rows = p.n_rows;
     g.out = static_cast<__nv_bfloat16*>(p.h); g.err = p.err;
     g.scale0 = p.s_gate; g.scale1 = p.s_up;
+    g.wait_limit_ns = wait_limit_ns();
     if ((err = launch_gemm(p.w_dtype, ma, mg, mu, oh, g, max_m * g.n_tiles, stream)) != cudaSuccess) return err;
 
     Params d = g;

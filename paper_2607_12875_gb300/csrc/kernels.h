@@ -51,6 +51,9 @@ size_t ffn_sched_ints(int E, int64_t n_rows);
 constexpr int64_t kDequantRowsPerExpert = 256;  // AUTO: TC_DEQUANT from this many rows per expert
 cudaError_t launch_ffn_stream(const FfnProblem& p, cudaStream_t stream);
 size_t stream_smem_bytes(int act_dtype, int H, int I);  // per CTA, streaming route
+// dynamic shared memory a CTA may use on sm_103a (227 KB); a streaming problem
+// runs when its stream_smem_bytes fits
+constexpr size_t stream_smem_budget() { return 227 * 1024; }
 cudaError_t launch_ffn_simt(const FfnProblem& p, cudaStream_t stream);
 cudaError_t launch_ffn_tc(const FfnProblem& p, cudaStream_t stream);
 bool ffn_tc_supported(const FfnProblem& p);

@@ -3,7 +3,9 @@
 // them into counts, offsets and per-block bases, and a scatter that ranks
 // pairs inside a block in pair order (warp match + warp-ordered running
 // counters), so the result is the stable order whatever the scheduling.
-// Up to 1024 pairs (decode) all three steps run in one CTA.
+// Up to 1024 pairs (decode) all three steps run in one CTA. A pair whose
+// expert id is outside [0, E) is dropped: pair_pos[p] = -1, and the sorted
+// positions past the last kept pair hold -1.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -75,7 +77,8 @@ perm_scan_kernel(const int32_t* __restrict__ block_hist, int nblk, int E, int32_
 
 __global__ void __launch_bounds__(kPermBlock)
 perm_scatter_kernel(const int32_t* __restrict__ ids, int64_t P, int E, const int32_t* __restrict__ block_base,
-                    int32_t* __restrict__ sorted_pair, int32_t* __restrict__ pair_pos) {
+                    const int32_t* __restrict__ offsets, int32_t* __restrict__ sorted_pair,
+                    int32_t* __restrict__ pair_pos) {
     pdl_enter();
     extern __shared__ int32_t s_run[];
     for (int e = threadIdx.x; e < E; e += blockDim.x) s_run[e] = block_base[(size_t)blockIdx.x * E + e];
@@ -101,7 +104,11 @@ perm_scatter_kernel(const int32_t* __restrict__ ids, int64_t P, int E, const int
     if (valid) {
         sorted_pair[pos] = (int32_t)p;
         pair_pos[p] = pos;
+    } else if (p < P) {
+        pair_pos[p] = -1;  // dropped pair: no slot
     }
+    // positions past the last kept pair (only when pairs were dropped) hold -1
+    if (p < P && p >= offsets[E]) sorted_pair[p] = -1;
 }
 
 // P <= kPermBlock: histogram, scan and stable scatter in one CTA (one pair
@@ -113,6 +120,7 @@ perm_small_kernel(const int32_t* __restrict__ ids, int64_t P, int E, int32_t* __
     pdl_enter();
     extern __shared__ int32_t s_run[];  // [E]: histogram, then running positions
     __shared__ int32_t s_warp[kPermBlock / 32];
+    __shared__ int32_t s_kept;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     for (int e = threadIdx.x; e < E; e += blockDim.x) s_run[e] = 0;
     __syncthreads();
@@ -145,7 +153,10 @@ perm_small_kernel(const int32_t* __restrict__ ids, int64_t P, int E, int32_t* __
     if (threadIdx.x < E) {
         counts[threadIdx.x] = cnt;
         offsets[threadIdx.x] = excl;
-        if (threadIdx.x == E - 1) offsets[E] = excl + cnt;
+        if (threadIdx.x == E - 1) {
+            offsets[E] = excl + cnt;
+            s_kept = excl + cnt;
+        }
         s_run[threadIdx.x] = excl;
     }
     __syncthreads();
@@ -165,7 +176,10 @@ perm_small_kernel(const int32_t* __restrict__ ids, int64_t P, int E, int32_t* __
     if (valid) {
         sorted_pair[pos] = p;
         pair_pos[p] = pos;
+    } else if (p < P) {
+        pair_pos[p] = -1;  // dropped pair: no slot
     }
+    if (p < P && p >= s_kept) sorted_pair[p] = -1;  // past the last kept pair
 }
 
 cudaError_t launch_permute(const int32_t* topk_ids, int64_t P, int E, int32_t* counts, int32_t* offsets,
@@ -189,7 +203,7 @@ cudaError_t launch_permute(const int32_t* topk_ids, int64_t P, int E, int32_t* c
     cudaError_t err = cudaGetLastError();
     if (err != cudaSuccess || nblk == 0) return err;
     if (const cudaError_t le = launch_k(perm_scatter_kernel, dim3(nblk), dim3(kPermBlock), E * sizeof(int32_t),
-            stream, topk_ids, P, E, block_base, sorted_pair, pair_pos); le != cudaSuccess)
+            stream, topk_ids, P, E, block_base, offsets, sorted_pair, pair_pos); le != cudaSuccess)
         return le;
     return cudaGetLastError();
 }

@@ -202,7 +202,8 @@ gate_logits_tiled_kernel(const __nv_bfloat16* __restrict__ x, const __nv_bfloat1
 // ------------------------------------------------------- expert choice
 
 // Fixed fp32 exponential for the sigmoid score (the expert choice depends on
-// its exact bits, so it is not left to a library): clamp to [-86, 88];
+// its exact bits, so it is not left to a library): NaN is returned as it
+// is, anything else clamped to [-86, 88];
 // n = rint(x*log2 e); r = (x - n*ln2_hi) - n*ln2_lo with ln2_hi the leading
 // 16 bits of ln 2 (Cody-Waite reduction, exact n*ln2_hi); exp(r) from its
 // degree-8 Taylor polynomial by Horner's rule, a separate rounded multiply
@@ -213,6 +214,7 @@ __device__ __forceinline__ float pinned_exp(float x) {
     const float kLn2Lo = __uint_as_float(0x35bfbe8eu);  // fp32(ln 2 - kLn2Hi)
     const uint32_t kInvFact[9] = {0x3f800000u, 0x3f800000u, 0x3f000000u, 0x3e2aaaabu, 0x3d2aaaabu,
                                   0x3c088889u, 0x3ab60b61u, 0x39500d01u, 0x37d00d01u};  // fp32(1/i!)
+    if (x != x) return x;  // NaN in, NaN out
     x = fminf(fmaxf(x, -86.0f), 88.0f);
     float n = rintf(__fmul_rn(x, kLog2e));
     float r = __fsub_rn(x, __fmul_rn(n, kLn2Hi));
@@ -227,10 +229,17 @@ __device__ __forceinline__ float pinned_sigmoid(float l) {
     return __fdiv_rn(1.0f, __fadd_rn(1.0f, pinned_exp(-l)));
 }
 
-// (key, index) with "larger key, then smaller index" as the better candidate
+// (key, index) with "larger key, then smaller index" as the better candidate.
+// Keys are never NaN here (choice_key), so this is a strict total order, and
+// a real candidate (index < kNone) beats an empty one even at key -inf.
+constexpr int kNone = 0x7fffffff;
 __device__ __forceinline__ bool better(float ka, int ia, float kb, int ib) {
     return ka > kb || (ka == kb && ia < ib);
 }
+
+// Key a score takes in the expert choice: a NaN counts as -infinity, so
+// non-finite logits still give valid, deterministic ids (ties to the lower index).
+__device__ __forceinline__ float choice_key(float v) { return v != v ? -INFINITY : v; }
 
 __device__ __forceinline__ void warp_best(float& k, int& i) {
 #pragma unroll
@@ -266,7 +275,7 @@ select_experts_kernel(const float* __restrict__ logits, const float* __restrict_
             sig[e] = s;
             v = select_bias ? __fadd_rn(s, select_bias[e]) : s;
         }
-        key[e] = v;
+        key[e] = choice_key(v);
     }
     __syncwarp();
 
@@ -282,15 +291,15 @@ select_experts_kernel(const float* __restrict__ logits, const float* __restrict_
                 float v = key[e];
                 if (v > a) { b = a; a = v; } else if (v > b) { b = v; }
             }
-            gscore = __fadd_rn(a, b);
+            gscore = choice_key(__fadd_rn(a, b));  // inf + -inf is NaN
         }
         kept = 0u;
         bool taken = false;
         for (int r = 0; r < rp.topk_group; ++r) {
             float kk = (lane < G && !taken) ? gscore : -INFINITY;
-            int ii = (lane < G && !taken) ? lane : 0x7fffffff;
+            int ii = (lane < G && !taken) ? lane : kNone;
             warp_best(kk, ii);
-            kept |= 1u << ii;
+            if (ii < 32) kept |= 1u << ii;  // always: topk_group <= G groups hold candidates
             if (lane == ii) taken = true;
         }
     }
@@ -302,17 +311,18 @@ select_experts_kernel(const float* __restrict__ logits, const float* __restrict_
     float top_key = 0.0f;
     for (int j = 0; j < k; ++j) {
         float kk = -INFINITY;
-        int ii = 0x7fffffff;
+        int ii = kNone;
         for (int s = 0, e = lane; e < E; ++s, e += 32) {
             if ((used >> s) & 1u) continue;
             if (!((kept >> (e / gs)) & 1u)) continue;
             float v = key[e];
-            if (ii == 0x7fffffff || better(v, e, kk, ii)) { kk = v; ii = e; }
+            if (ii == kNone || better(v, e, kk, ii)) { kk = v; ii = e; }
         }
         warp_best(kk, ii);
-        if ((ii & 31) == lane) used |= 1u << (ii >> 5);
+        // ii < E always (check_config keeps top_k within the kept groups' experts)
+        if (ii < E && (ii & 31) == lane) used |= 1u << (ii >> 5);
         if (j == 0) top_key = kk;
-        if (lane == j) sel_id = ii;
+        if (lane == j) sel_id = ii < E ? ii : 0;
     }
 
     // routing weights (lane j < k holds slot j)
@@ -356,8 +366,11 @@ cudaError_t launch_route(const RouteParams& rp, const void* x, const void* wg, c
         auto xp = static_cast<const __nv_bfloat16*>(x);
         auto wp = static_cast<const __nv_bfloat16*>(wg);
         if (rp.T >= 1024) {
-            cudaError_t e = cudaFuncSetAttribute(gate_logits_tiled_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 (int)kGateTiledSmem);
+            static DeviceOnce smem_set;
+            cudaError_t e = smem_set.run([] {
+                return cudaFuncSetAttribute(gate_logits_tiled_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                            (int)kGateTiledSmem);
+            });
             if (e != cudaSuccess) return e;
             dim3 grid((rp.T + kGT - 1) / kGT, (rp.E + kGE - 1) / kGE);
             if (const cudaError_t le = launch_k(gate_logits_tiled_kernel, dim3(grid), dim3(256), kGateTiledSmem,

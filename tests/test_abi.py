@@ -138,3 +138,23 @@ def test_dequant_route_workspace_holds_bf16_weight_copies(lib, wid):
     dq = gb.workspace_size(cfg_of(wid, ffn_route=gb.FFN_TC_DEQUANT))
     copies = 3 * wl.E * wl.H * wl.I * 2 + (3 * wl.H * wl.I_shared * 2 if wl.has_shared else 0)
     assert copies <= dq - tc <= copies + 2 * 256
+
+
+def test_forced_stream_route_checks_the_shared_expert_before_launching(lib):
+    """With both FFN problems forced onto the streaming route, a shared expert
+    whose rows do not fit the streaming kernel's shared memory is refused
+    before anything is enqueued (the routed problem alone would fit)."""
+    c = cfg_of(4, T=4, ffn_route=gb.FFN_STREAM, I_shared=16384)
+    assert gb.check_config(c) == gb.OK
+    assert gb.ffn_route(c) == "stream" and gb.ffn_route(c, shared=True) == "stream"
+    p = FakePtr()
+    ws = FakePtr(gb.workspace_size(c))
+    w = gb.weights(p, p, p, p, p, p)
+    with pytest.raises(gb.GbmoeError) as e:
+        gb.moe_forward(c, p, p, None, None, w, w, p, ws, stream=0)
+    assert e.value.status == gb.EUNSUPPORTED
+    with pytest.raises(gb.GbmoeError) as e:
+        gb.moe_shared_ffn(c, p, w, p, ws, stream=0)
+    assert e.value.status == gb.EUNSUPPORTED
+    c.I_shared = 2048  # fits: the same call passes the checks (it would launch, so it is not made here)
+    assert gb.check_config(c) == gb.OK
