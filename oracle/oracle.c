@@ -335,11 +335,30 @@ double oracle_e4m3_value(uint8_t code) {
 
 /* Dequantised weight of one [N, K] expert matrix stored as e4m3 codes with
  * one fp32 scale per 128x128 block: W[n,k] = e4m3(q[n,k]) * s[n/128][k/128],
- * exact in fp64. */
-void oracle_dequant_fp8_b128(int64_t N, int64_t K, const uint8_t* q, const float* s, double* out) {
-    for (int64_t n = 0; n < N; ++n)
+ * exact in fp64 (a 4-bit by 24-bit significand product). The 256 code values
+ * are taken from oracle_e4m3_value once per call; rows are independent and
+ * shared out over threads. */
+typedef struct {
+    int64_t K;
+    const uint8_t* q;
+    const float* s;
+    double* out;
+    double value[256];
+} fp8_ctx;
+
+static void fp8_rows(void* vp, int64_t b, int64_t e) {
+    fp8_ctx* c = (fp8_ctx*)vp;
+    const int64_t K = c->K;
+    for (int64_t n = b; n < e; ++n)
         for (int64_t k = 0; k < K; ++k)
-            out[n * K + k] = oracle_e4m3_value(q[n * K + k]) * (double)s[(n / 128) * (K / 128) + k / 128];
+            c->out[n * K + k] = c->value[c->q[n * K + k]] * (double)c->s[(n / 128) * (K / 128) + k / 128];
+}
+
+void oracle_dequant_fp8_b128(int64_t N, int64_t K, const uint8_t* q, const float* s, double* out) {
+    fp8_ctx c;
+    c.K = K; c.q = q; c.s = s; c.out = out;
+    for (int code = 0; code < 256; ++code) c.value[code] = oracle_e4m3_value((uint8_t)code);
+    parallel_for(N, fp8_rows, &c);
 }
 
 static double bf16_value(uint16_t h) { return (double)f32_from_bits((uint32_t)h << 16); }
@@ -347,15 +366,29 @@ static double bf16_value(uint16_t h) { return (double)f32_from_bits((uint32_t)h 
 /* Dequantised weight of one [N, K] expert matrix stored as symmetric int4
  * (two's complement nibble, element 2i in the low nibble of byte i of a row)
  * with one bf16 scale per 128 consecutive k: W[n,k] = q[n,k] * s[n][k/128],
- * exact in fp64. */
-void oracle_dequant_int4_g128(int64_t N, int64_t K, const uint8_t* q, const uint16_t* s, double* out) {
-    for (int64_t n = 0; n < N; ++n)
+ * exact in fp64. Rows are shared out over threads. */
+typedef struct {
+    int64_t K;
+    const uint8_t* q;
+    const uint16_t* s;
+    double* out;
+} int4_ctx;
+
+static void int4_rows(void* vp, int64_t b, int64_t e) {
+    int4_ctx* c = (int4_ctx*)vp;
+    const int64_t K = c->K;
+    for (int64_t n = b; n < e; ++n)
         for (int64_t k = 0; k < K; ++k) {
-            uint8_t byte = q[n * (K / 2) + k / 2];
+            uint8_t byte = c->q[n * (K / 2) + k / 2];
             int v = (k % 2 == 0) ? (byte & 0xf) : (byte >> 4);
             if (v >= 8) v -= 16;
-            out[n * K + k] = (double)v * bf16_value(s[n * (K / 128) + k / 128]);
+            c->out[n * K + k] = (double)v * bf16_value(c->s[n * (K / 128) + k / 128]);
         }
+}
+
+void oracle_dequant_int4_g128(int64_t N, int64_t K, const uint8_t* q, const uint16_t* s, double* out) {
+    int4_ctx c = {K, q, s, out};
+    parallel_for(N, int4_rows, &c);
 }
 
 void oracle_pexp_n(int64_t n, const float* in, float* out) {
@@ -366,57 +399,29 @@ void oracle_sigmoid_n(int64_t n, const float* in, float* out) {
     for (int64_t i = 0; i < n; ++i) out[i] = oracle_sigmoid(in[i]);
 }
 
+typedef struct {
+    const void* in;
+    double* out;
+} widen_ctx;
+
+static void widen_f32_range(void* vp, int64_t b, int64_t e) {
+    widen_ctx* c = (widen_ctx*)vp;
+    for (int64_t i = b; i < e; ++i) c->out[i] = (double)((const float*)c->in)[i];
+}
+
+static void widen_bf16_range(void* vp, int64_t b, int64_t e) {
+    widen_ctx* c = (widen_ctx*)vp;
+    for (int64_t i = b; i < e; ++i) c->out[i] = bf16_value(((const uint16_t*)c->in)[i]);
+}
+
 void oracle_widen_f32(int64_t n, const float* in, double* out) {
-    for (int64_t i = 0; i < n; ++i) out[i] = (double)in[i];
+    widen_ctx c = {in, out};
+    parallel_for(n, widen_f32_range, &c);
 }
 
 void oracle_widen_bf16(int64_t n, const uint16_t* in, double* out) {
-    for (int64_t i = 0; i < n; ++i) out[i] = bf16_value(in[i]);
-}
-
-/* ============================== Fused MoE: one expert's SwiGLU FFN */
-
-/*
- * For each of n_rows activation rows x (fp64, length H) routed to one expert:
- *   g = Wgate x,  u = Wup x            (Wgate, Wup: [I, H])
- *   a_i = silu(g_i) * u_i,  silu(z) = z / (1 + exp(-z))
- *   y = Wdown a                        (Wdown: [H, I])
- * all in fp64. The expert FFN is the standard gated (SwiGLU) MLP of the
- * MoE models the paper serves (Section 6); the paper does not print it.
- */
-typedef struct {
-    int64_t H, I;
-    const double *x, *wg, *wu, *wd;
-    double* y;
-} ffn_ctx;
-
-static void ffn_range(void* vp, int64_t b, int64_t e) {
-    ffn_ctx* c = (ffn_ctx*)vp;
-    double* a = (double*)malloc(sizeof(double) * c->I);
-    for (int64_t r = b; r < e; ++r) {
-        const double* x = c->x + r * c->H;
-        for (int64_t i = 0; i < c->I; ++i) {
-            double g = 0.0, u = 0.0;
-            for (int64_t h = 0; h < c->H; ++h) {
-                g += c->wg[i * c->H + h] * x[h];
-                u += c->wu[i * c->H + h] * x[h];
-            }
-            a[i] = g / (1.0 + exp(-g)) * u;
-        }
-        double* y = c->y + r * c->H;
-        for (int64_t n = 0; n < c->H; ++n) {
-            double acc = 0.0;
-            for (int64_t i = 0; i < c->I; ++i) acc += c->wd[n * c->I + i] * a[i];
-            y[n] = acc;
-        }
-    }
-    free(a);
-}
-
-void oracle_expert_ffn(int64_t n_rows, int64_t H, int64_t I, const double* x, const double* w_gate,
-                       const double* w_up, const double* w_down, double* y) {
-    ffn_ctx c = {H, I, x, w_gate, w_up, w_down, y};
-    parallel_for(n_rows, ffn_range, &c);
+    widen_ctx c = {in, out};
+    parallel_for(n, widen_bf16_range, &c);
 }
 
 /* ==================================================== Weight Sum */
@@ -426,14 +431,28 @@ void oracle_expert_ffn(int64_t n_rows, int64_t H, int64_t I, const double* x, co
  *            (+ y_shared[t,:] when a shared expert is present, weight 1),
  * in fp64. y_pairs holds one expert output row per sorted pair position.
  */
-void oracle_combine(int64_t T, int64_t k, int64_t H, const double* y_pairs, const double* w,
-                    const int32_t* pair_pos, const double* y_shared, double* out) {
-    for (int64_t t = 0; t < T; ++t)
+typedef struct {
+    int64_t k, H;
+    const double *y_pairs, *w, *y_shared;
+    const int32_t* pair_pos;
+    double* out;
+} combine_ctx;
+
+static void combine_range(void* vp, int64_t b, int64_t e) {
+    combine_ctx* c = (combine_ctx*)vp;
+    const int64_t k = c->k, H = c->H;
+    for (int64_t t = b; t < e; ++t)
         for (int64_t h = 0; h < H; ++h) {
             double acc = 0.0;
             for (int64_t j = 0; j < k; ++j)
-                acc += w[t * k + j] * y_pairs[(int64_t)pair_pos[t * k + j] * H + h];
-            if (y_shared) acc += y_shared[t * H + h];
-            out[t * H + h] = acc;
+                acc += c->w[t * k + j] * c->y_pairs[(int64_t)c->pair_pos[t * k + j] * H + h];
+            if (c->y_shared) acc += c->y_shared[t * H + h];
+            c->out[t * H + h] = acc;
         }
+}
+
+void oracle_combine(int64_t T, int64_t k, int64_t H, const double* y_pairs, const double* w,
+                    const int32_t* pair_pos, const double* y_shared, double* out) {
+    combine_ctx c = {k, H, y_pairs, w, y_shared, pair_pos, out};
+    parallel_for(T, combine_range, &c);
 }
