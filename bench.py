@@ -5,11 +5,14 @@
 
 A step is one full layer forward (MoE Gate, permutation, expert FFNs,
 Weight Sum) over one batch of the workload, through the C ABI (moe_forward)
-on inputs already resident in HBM. The default workload is the decode-shaped
-bf16 layer: T=32 tokens, hidden 4096, 128 experts, top-8, intermediate 1536.
-Its active experts' weights (~4.2 GB) exceed the 126 MB L2, so no flush is
-needed between steps. With N GPUs (torchrun) every rank runs its own replica
-on its own batch (the layer has no exchange step here): weak scaling.
+on inputs already resident in HBM. The headline workload is the decode-shaped
+bf16 layer: T=32 tokens, hidden 4096, 128 experts, top-8, intermediate 1536;
+the same line carries, under per_config, the same measurements for the
+prefill bf16 (T=8192), DeepSeek-style fp8 (T=2048, 256 + 1 experts) and
+skewed int4 (T=16384) layers. Every workload's active expert weights (1.1 GB
+and up) exceed the 126 MB L2, so no flush is needed between steps. With N
+GPUs (torchrun) every rank runs its own replica on its own batch (the layer
+has no exchange step here): weak scaling.
 
 --impl reference times the CPU oracle (test infrastructure, plain C) on the
 host cores on a bounded token sample of the same workload.
@@ -240,51 +243,50 @@ def workload_config(wl):
             "l2": "no flush: the active experts' weights read each step exceed the 126 MB L2"}
 
 
-def main():
-    ap = argparse.ArgumentParser()
-    ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=200)
-    ap.add_argument("--warmup", type=int, default=10)
-    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--workload", type=int, default=2, help="synth.WORKLOADS id (2 = decode bf16)")
-    ap.add_argument("--route", default="auto", choices=["auto", "stream", "simt", "tc", "tc_dequant"])
-    ap.add_argument("--ref-tokens", type=int, default=1, help="tokens per oracle step (reference arm)")
-    ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--set", action="append", default=[], metavar="KEY=INT",
-                    help="override a workload field (reduced cases for profiling), e.g. --set T=2048 --set E=32")
-    ap.add_argument("--profile", type=int, default=0, metavar="N",
-                    help="run N untimed layer forwards and exit (for ncu captures); prints no bench line")
-    args = ap.parse_args()
-    if args.warmup < 3 and args.impl == "ours":
-        args.warmup = 3
+def launches_per_step(wl, route: str, shared_route) -> int:
+    """Kernels this library launches per layer forward: gate logits + expert
+    choice, the permutation (one kernel up to 1024 pairs, else three), per FFN
+    problem a schedule kernel + 2 GEMM/stream kernels (+ a row gather for the
+    routed experts on the tensor-core routes, + 3 weight-decode passes on the
+    decode-once route), and the combine."""
+    def ffn(r, routed):
+        return 3 + (1 if routed and r in ("tc", "tc_dequant") else 0) + (3 if r == "tc_dequant" else 0)
 
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
+    n = 2 + (1 if wl.P <= 1024 else 3) + ffn(route, True) + 1
+    if shared_route is not None:
+        n += ffn(shared_route, False)
+    return n
 
-    if args.impl == "reference":
-        if rank != 0:
-            return
-        wl, inp = load_workload(args.workload, args.set)
-        print(json.dumps(run_reference(args, wl, inp, rank)))
-        return
 
+def cpu_baseline_entry(wl, inp) -> dict:
+    """The oracle on the host cores: the first 32 tokens (full routing of every
+    token plus those tokens' expert FFNs and combine), repeated until about
+    10 s of work (at most 8 runs)."""
+    import oracle
+
+    n_tok = min(wl.T, 32)
+    dt, runs = 0.0, 0
+    while runs == 0 or (dt < 10.0 and runs < 8):
+        t0 = time.perf_counter()
+        oracle.forward(wl, inp, rows=list(range(n_tok)))
+        dt += time.perf_counter() - t0
+        runs += 1
+    return {"value": n_tok * runs / dt, "unit": "tokens/s", "cores": oracle.get_threads(), "kind": "oracle",
+            "sample": f"first {n_tok} tokens, {runs} runs: full routing of all {wl.T} tokens plus the expert "
+                      f"FFNs and combine of the sampled ones ({dt:.1f} s)"}
+
+
+def measure(args, wid: int, overrides, dist, world: int, rank: int, local: int, with_cpu: bool) -> dict | None:
+    """One workload: the layer timed over args.steps forwards (CUDA events on
+    the launching stream, clocks sampled meanwhile), the expert FFN timed
+    alone for the roofline, the host-buffer entry point end to end, and
+    (rank 0, one GPU) the oracle on the host cores. Returns the bench fields
+    (None for --profile runs)."""
     import torch
 
     import paper_2607_12875_gb300 as gb
 
-    torch.cuda.set_device(local)
-    dist = None
-    if world > 1:
-        import torch.distributed as dist
-
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
-
-    def barrier():
-        if dist is not None:
-            dist.barrier()
-
-    wl, inp = load_workload(args.workload, args.set)
+    wl, inp = load_workload(wid, overrides)
     dev = torch.device("cuda", local)
 
     def act(a):
@@ -297,6 +299,10 @@ def main():
         for k, v in store.items():
             d[k] = torch.from_numpy(v.view(np.int16) if v.dtype == np.uint16 else v).to(dev)
         return gb.weights(d["w_gate"], d["w_up"], d["w_down"], d.get("s_gate"), d.get("s_up"), d.get("s_down")), d
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
 
     x = act(inp["x"])
     wr = act(inp["w_router"])
@@ -319,8 +325,8 @@ def main():
         for _ in range(args.profile):
             step()
         torch.cuda.synchronize()
-        print(f"profile run: {wl.name} {args.set} route={gb.ffn_route(cfg)} status={gb.moe_device_status(ws)}")
-        return
+        print(f"profile run: {wl.name} {overrides} route={gb.ffn_route(cfg)} status={gb.moe_device_status(ws)}")
+        return None
 
     for _ in range(args.warmup):
         step()
@@ -368,6 +374,7 @@ def main():
     fe.record(stream)
     torch.cuda.synchronize()
     ffn_ms = fs.elapsed_time(fe) / args.steps
+    del y
     pk, pk_kind = peaks()
     route = gb.ffn_route(cfg)
     # the expert FFN's roofline: the slower of its algorithmic weight bytes over
@@ -380,7 +387,8 @@ def main():
                             "gate/up GEMM with SwiGLU + down GEMM)",
               "simt": "moe_grouped_ffn, CUDA-core route"}[route]
     tpe = TRAFFIC_PER_ACTIVE_EXPERT.get((wl.name, route))
-    extra = {"traffic": None if tpe is None else tpe * active, "kernel": kernel, "active_experts": active}
+    extra = {"traffic": None if tpe is None else tpe * active, "kernel": kernel, "active_experts": active,
+             "route": route}
     roofline = roofline_entry(routed_bytes, flops, ffn_ms, pk, pk_kind, extra)
 
     # end to end through the public host-buffer entry point
@@ -399,43 +407,85 @@ def main():
     e2e_s = max_over_ranks(e2e_s, dist, dev)
     io_bytes = wl.T * wl.H * x.element_size()
     e2e = {"value": replica_throughput(wl.T, args.steps, world, e2e_s), "unit": "tokens/s",
-           "h2d_bytes_per_step": io_bytes,
-           "d2h_bytes_per_step": io_bytes}
+           "h2d_bytes_per_step": io_bytes, "d2h_bytes_per_step": io_bytes}
 
-    # kernels this library launched per step: gate logits + expert choice, 3 for the
-    # permutation (one up to 1024 pairs), per FFN problem a schedule kernel + 2 (+ a row
-    # gather for the routed experts on the tensor-core routes, + 3 weight-decode passes on
-    # the decode-once route), combine
-    def ffn_launches(r, routed):
-        return 3 + (1 if routed and r in ("tc", "tc_dequant") else 0) + (3 if r == "tc_dequant" else 0)
+    per_step = launches_per_step(wl, route, gb.ffn_route(cfg, shared=True) if wl.has_shared else None)
+    cpu = cpu_baseline_entry(wl, inp) if with_cpu else None
+    del x, wr, lb, sb, experts, shared, keep1, keep2, ws, out, x_host, out_host
+    torch.cuda.empty_cache()
+    return {"value": value, "ms_per_step": ms / args.steps, "steps": args.steps,
+            "dtype": wl.act if wl.wq in ("f32", "bf16") else f"{wl.act}+{wl.wq}",
+            "config": workload_config(wl), "clocks": clocks.summary(), "e2e": e2e,
+            "gpu_launches": per_step * args.steps, "roofline": roofline, "cpu_baseline": cpu}
 
-    per_step = 2 + (1 if wl.P <= 1024 else 3) + ffn_launches(route, True) + 1
-    if wl.has_shared:
-        per_step += ffn_launches(gb.ffn_route(cfg, shared=True), False)
 
-    cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        import oracle
+# workloads the default run times besides the headline one: prefill bf16,
+# DeepSeek-style fp8 and skewed int4 (the benchmark spec's other size classes)
+PER_CONFIG = (3, 4, 5)
 
-        # the first 32 tokens, repeated until about 10 s of oracle work (at most 8 runs)
-        n_tok = min(wl.T, 32)
-        dt, runs = 0.0, 0
-        while runs == 0 or (dt < 10.0 and runs < 8):
-            t0 = time.perf_counter()
-            oracle.forward(wl, inp, rows=list(range(n_tok)))
-            dt += time.perf_counter() - t0
-            runs += 1
-        cpu = {"value": n_tok * runs / dt, "unit": "tokens/s", "cores": oracle.get_threads(), "kind": "oracle",
-               "sample": f"first {n_tok} tokens, {runs} runs: full routing of all {wl.T} tokens plus the expert "
-                         f"FFNs and combine of the sampled ones ({dt:.1f} s)"}
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", type=int, default=2, help="synth.WORKLOADS id of the headline (2 = decode bf16)")
+    ap.add_argument("--route", default="auto", choices=["auto", "stream", "simt", "tc", "tc_dequant"])
+    ap.add_argument("--ref-tokens", type=int, default=1, help="tokens per oracle step (reference arm)")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-per-config", action="store_true",
+                    help="time only the headline workload (by default workloads 3, 4 and 5 are timed too)")
+    ap.add_argument("--set", action="append", default=[], metavar="KEY=INT",
+                    help="override a workload field (reduced cases for profiling), e.g. --set T=2048 --set E=32")
+    ap.add_argument("--profile", type=int, default=0, metavar="N",
+                    help="run N untimed layer forwards and exit (for ncu captures); prints no bench line")
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "ours":
+        args.warmup = 3
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        wl, inp = load_workload(args.workload, args.set)
+        print(json.dumps(run_reference(args, wl, inp, rank)))
+        return
+
+    import torch
+
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+
+    with_cpu = rank == 0 and world == 1 and not args.no_cpu_baseline
+    head = measure(args, args.workload, args.set, dist, world, rank, local, with_cpu)
+    if head is None:  # --profile
+        return
+    per_config = {}
+    if not args.no_per_config and not args.set and args.route == "auto":
+        for wid in PER_CONFIG:
+            if wid == args.workload:
+                continue
+            m = measure(args, wid, (), dist, world, rank, local, with_cpu)
+            per_config[m["config"]["workload"]] = {"value": m["value"], "unit": "tokens/s", "n_gpus": world, **m}
 
     if rank == 0:
-        line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
-                "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
-                "vs_baseline": None, "dtype": wl.act if wl.wq in ("f32", "bf16") else f"{wl.act}+{wl.wq}",
+        line = {"metric": METRIC, "value": head["value"], "unit": "tokens/s", "n_gpus": world,
+                "steps": args.steps, "warmup": args.warmup, "ms_per_step": head["ms_per_step"],
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": head["dtype"],
                 "data": "synthetic (seeded SplitMix64/Irwin-Hall normals; random-init weights)",
-                "config": workload_config(wl), "clocks": clocks.summary(), "e2e": e2e,
-                "gpu_launches": per_step * args.steps, "roofline": roofline, "cpu_baseline": cpu}
+                "config": head["config"], "clocks": head["clocks"], "e2e": head["e2e"],
+                "gpu_launches": head["gpu_launches"], "roofline": head["roofline"],
+                "cpu_baseline": head["cpu_baseline"]}
+        if per_config:
+            line["per_config"] = per_config
         print(json.dumps(line))
     if dist is not None:
         dist.destroy_process_group()

@@ -83,15 +83,45 @@ def rel_err(got: np.ndarray, ref: np.ndarray) -> float:
     return float(np.max(np.abs(got - ref)) / max(np.max(np.abs(ref)), 1e-30))
 
 
-def sample_rows(wl, ids: np.ndarray, n_random: int, per_extreme: int, seed: int = 0) -> np.ndarray:
-    """Seeded token subset: random tokens, the first and last token, and up to
-    per_extreme tokens routed to the hottest and to the coldest active expert."""
-    rng = np.random.default_rng(seed)
-    T = ids.shape[0]
-    rows = set(rng.choice(T, size=min(n_random, T), replace=False).tolist()) | {0, T - 1}
-    counts = np.bincount(ids.ravel(), minlength=wl.E)
-    active = np.nonzero(counts)[0]
-    for e in (active[np.argmax(counts[active])], active[np.argmin(counts[active])]):
-        toks = np.nonzero((ids == e).any(axis=1))[0]
-        rows |= set(rng.choice(toks, size=min(per_extreme, len(toks)), replace=False).tolist())
-    return np.array(sorted(rows), dtype=np.int64)
+ROW_FLOOR = 0.05  # per-row errors are taken relative to max(|ref row|, ROW_FLOOR * max |ref|)
+
+
+def error_report(got: np.ndarray, ref: np.ndarray) -> dict:
+    """Errors of got against ref over rows (the last axis is a row's elements):
+    the infinity-norm relative error (the tolerance metric), per-row relative
+    errors max|got_r - ref_r| / max(max|ref_r|, ROW_FLOOR * max|ref|), and the
+    largest elementwise relative error with the same floor."""
+    got = got.reshape(-1, got.shape[-1])
+    ref = ref.reshape(-1, ref.shape[-1])
+    gmax = max(float(np.max(np.abs(ref))), 1e-30)
+    diff = np.abs(got - ref)
+    row_scale = np.maximum(np.max(np.abs(ref), axis=1), ROW_FLOOR * gmax)
+    row_err = np.max(diff, axis=1) / row_scale
+    elem_err = diff / np.maximum(np.abs(ref), ROW_FLOOR * gmax)
+    worst = np.argsort(row_err)[::-1][:3]
+    return {"inf": float(np.max(diff) / gmax), "row_max": float(np.max(row_err)),
+            "row_median": float(np.median(row_err)), "worst_rows": [(int(r), float(row_err[r])) for r in worst],
+            "elem_max": float(np.max(elem_err)), "rows": int(got.shape[0])}
+
+
+def assert_close(got: np.ndarray, ref: np.ndarray, tol: float, what: str = "output") -> dict:
+    """The infinity-norm relative error and every per-row relative error
+    within tol; the report (worst rows, elementwise error) is the message."""
+    rep = error_report(got, ref)
+    assert rep["inf"] <= tol and rep["row_max"] <= tol, f"{what}: {rep} (tol {tol:.0e})"
+    return rep
+
+
+def tiles_covered(ids_rows: np.ndarray, rows: np.ndarray, counts: np.ndarray, sorted_pair: np.ndarray,
+                  offsets: np.ndarray, bm: int = 128) -> tuple:
+    """(covered, total): how many of the (expert, bm-row tile) pairs of the
+    grouped GEMM hold at least one pair of the compared tokens `rows`."""
+    k = ids_rows.shape[1]
+    want = set(rows.tolist())
+    total, covered = 0, 0
+    for e in np.nonzero(counts)[0]:
+        for m in range(0, int(counts[e]), bm):
+            total += 1
+            seg = sorted_pair[offsets[e] + m: offsets[e] + min(m + bm, int(counts[e]))] // k
+            covered += bool(want.intersection(seg.tolist()))
+    return covered, total
