@@ -154,6 +154,8 @@ def expert_bytes(wq: str, H: int, I: int) -> int:
         return per * 4
     if wq == "fp8_b128":  # e4m3 codes + one fp32 scale per 128x128 block
         return per + 3 * (H // 128) * (I // 128) * 4
+    if wq == "mxfp4":  # E2M1 nibbles + one E8M0 byte per 32 along K
+        return per // 2 + 3 * (H * I // 32)
     return per // 2 + 3 * (H * I // 128) * 2  # int4 nibbles + one bf16 scale per 128 along K
 
 
@@ -420,8 +422,9 @@ def measure(args, wid: int, overrides, dist, world: int, rank: int, local: int, 
 
 
 # workloads the default run times besides the headline one: prefill bf16,
-# DeepSeek-style fp8 and skewed int4 (the benchmark spec's other size classes)
-PER_CONFIG = (3, 4, 5)
+# DeepSeek-style fp8 and skewed int4 (the benchmark spec's other size classes),
+# and the DeepSeek-style layer with MXFP4 experts
+PER_CONFIG = (3, 4, 5, 6)
 
 
 def main():

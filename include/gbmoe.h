@@ -51,12 +51,13 @@ enum {
     GBMOE_EDEVICE_TIMEOUT = -5  /* a bounded device-side wait gave up           */
 };
 
-/* Element types. act_dtype uses F32 or BF16; w_dtype any of the four. */
+/* Element types. act_dtype uses F32 or BF16; w_dtype any of the five. */
 enum {
     GBMOE_F32 = 0,
     GBMOE_BF16 = 1,
     GBMOE_FP8_E4M3_B128 = 2, /* e4m3 codes + fp32 scale per 128x128 block      */
-    GBMOE_INT4_G128 = 3      /* packed int4 + bf16 scale per 128 along K (row) */
+    GBMOE_INT4_G128 = 3,     /* packed int4 + bf16 scale per 128 along K (row) */
+    GBMOE_MXFP4 = 4          /* packed FP4 E2M1 + E8M0 scale per 32 along K    */
 };
 
 /* Router scoring. */
@@ -65,7 +66,7 @@ enum { GBMOE_SOFTMAX = 0, GBMOE_SIGMOID = 1 };
 /* Which expert-FFN kernels run. AUTO streams weights when the average number
  * of rows per expert P/E is at most 16 and otherwise runs the grouped GEMM
  * (tensor cores for bf16 activations, CUDA cores for fp32). On the tensor
- * cores, fp8/int4 weights are decoded inside the GEMM when P/E < 256; with
+ * cores, fp8/int4/MXFP4 weights are decoded inside the GEMM when P/E < 256; with
  * more rows per expert (several M tiles reuse each weight tile) AUTO takes
  * GBMOE_FFN_TC_DEQUANT: one pass decodes the active experts' weights to a
  * bf16 copy in the workspace (the same bf16 values the in-GEMM decode makes),
@@ -102,7 +103,15 @@ typedef struct gbmoe_config {
  *  INT4_G128:       w_* hold packed nibbles, [E, N, K/2] bytes for an [N, K]
  *                   matrix, element 2i in the low nibble of byte i, two's
  *                   complement; s_* are bf16 [E, N, K/128];
- *                   W[n,k] = q[n,k] * s[n][k/128]. */
+ *                   W[n,k] = q[n,k] * s[n][k/128].
+ *  MXFP4:           the OCP Microscaling FP4 format, the MXFP4 expert weights
+ *                   of the DeepSeek reference path (Section 6.2): w_* hold
+ *                   packed FP4 E2M1 nibbles laid out as for INT4_G128 (sign in
+ *                   bit 3, 2 exponent bits with bias 1, 1 mantissa bit:
+ *                   0, 0.5, 1, 1.5, 2, 3, 4, 6); s_* are E8M0 bytes
+ *                   [E, N, K/32], 2-byte aligned;
+ *                   W[n,k] = e2m1(q[n,k]) * 2^(s[n][k/32] - 127). Decoding
+ *                   to bf16 or fp32 is exact. */
 typedef struct gbmoe_expert_weights {
     const void *w_gate, *w_up, *w_down;
     const void *s_gate, *s_up, *s_down;

@@ -66,6 +66,11 @@ def _L():
         lib.oracle_e4m3_value.restype = ctypes.c_double
         lib.oracle_dequant_fp8_b128.argtypes = [i64, i64, vp, vp, vp]
         lib.oracle_dequant_int4_g128.argtypes = [i64, i64, vp, vp, vp]
+        lib.oracle_e2m1_value.argtypes = [ctypes.c_uint8]
+        lib.oracle_e2m1_value.restype = ctypes.c_double
+        lib.oracle_e8m0_value.argtypes = [ctypes.c_uint8]
+        lib.oracle_e8m0_value.restype = ctypes.c_double
+        lib.oracle_dequant_mxfp4.argtypes = [i64, i64, vp, vp, vp]
         lib.oracle_widen_f32.argtypes = [i64, vp, vp]
         lib.oracle_widen_bf16.argtypes = [i64, vp, vp]
         lib.oracle_combine.argtypes = [i64, i64, i64, vp, vp, vp, vp, vp]
@@ -176,6 +181,23 @@ def dequant_int4_g128(q: np.ndarray, s: np.ndarray) -> np.ndarray:
     return out
 
 
+def e2m1_value(code: int) -> float:
+    return _L().oracle_e2m1_value(code)
+
+
+def e8m0_value(code: int) -> float:
+    return _L().oracle_e8m0_value(code)
+
+
+def dequant_mxfp4(q: np.ndarray, s: np.ndarray) -> np.ndarray:
+    q = _c(q, np.uint8)
+    s = _c(s, np.uint8)
+    N, K2 = q.shape
+    out = np.empty((N, 2 * K2), np.float64)
+    _L().oracle_dequant_mxfp4(N, 2 * K2, _p(q), _p(s), _p(out))
+    return out
+
+
 def widen(a: np.ndarray, dtype: str) -> np.ndarray:
     """Exact fp64 copy of fp32 values or of raw bf16 bit patterns."""
     if dtype == "f32":
@@ -198,6 +220,8 @@ def weight_f64(store: dict, name: str, e: int, wq: str) -> np.ndarray:
         return dequant_fp8_b128(q, store["s_" + name][e])
     if wq == "int4_g128":
         return dequant_int4_g128(q, store["s_" + name][e])
+    if wq == "mxfp4":
+        return dequant_mxfp4(q, store["s_" + name][e])
     raise ValueError(wq)
 
 

@@ -391,6 +391,51 @@ void oracle_dequant_int4_g128(int64_t N, int64_t K, const uint8_t* q, const uint
     parallel_for(N, int4_rows, &c);
 }
 
+/*
+ * MXFP4 (OCP Microscaling Formats v1.0): the MXFP4 expert weights of the
+ * DeepSeek reference path (Section 6.2). Each element is FP4 E2M1: sign bit 3,
+ * a 2-bit exponent with bias 1 (bits 2-1) and one mantissa bit (bit 0);
+ * exponent 0 is subnormal, m * 0.5; no infinities or NaN. Each block of 32
+ * consecutive k shares an E8M0 scale: 2^(s - 127), s = 255 being NaN.
+ */
+double oracle_e2m1_value(uint8_t code) {
+    int sign = (code >> 3) & 1, ex = (code >> 1) & 3, m = code & 1;
+    double v = ex == 0 ? 0.5 * m : ldexp(1.0 + 0.5 * m, ex - 1);
+    return sign ? -v : v;
+}
+
+double oracle_e8m0_value(uint8_t s) { return s == 255 ? NAN : ldexp(1.0, (int)s - 127); }
+
+/* Dequantised weight of one [N, K] expert matrix stored as MXFP4: element
+ * 2i in the low nibble of byte i of a row, scale s[n][k/32]:
+ * W[n,k] = e2m1(q[n,k]) * 2^(s[n][k/32] - 127), exact in fp64. Rows are
+ * shared out over threads. */
+typedef struct {
+    int64_t K;
+    const uint8_t* q;
+    const uint8_t* s;
+    double* out;
+    double value[16];
+} mxfp4_ctx;
+
+static void mxfp4_rows(void* vp, int64_t b, int64_t e) {
+    mxfp4_ctx* c = (mxfp4_ctx*)vp;
+    const int64_t K = c->K;
+    for (int64_t n = b; n < e; ++n)
+        for (int64_t k = 0; k < K; ++k) {
+            uint8_t byte = c->q[n * (K / 2) + k / 2];
+            int code = (k % 2 == 0) ? (byte & 0xf) : (byte >> 4);
+            c->out[n * K + k] = c->value[code] * oracle_e8m0_value(c->s[n * (K / 32) + k / 32]);
+        }
+}
+
+void oracle_dequant_mxfp4(int64_t N, int64_t K, const uint8_t* q, const uint8_t* s, double* out) {
+    mxfp4_ctx c;
+    c.K = K; c.q = q; c.s = s; c.out = out;
+    for (int code = 0; code < 16; ++code) c.value[code] = oracle_e2m1_value((uint8_t)code);
+    parallel_for(N, mxfp4_rows, &c);
+}
+
 void oracle_pexp_n(int64_t n, const float* in, float* out) {
     for (int64_t i = 0; i < n; ++i) out[i] = oracle_pexp(in[i]);
 }

@@ -17,11 +17,11 @@ LIB_PATH = os.path.join(_HERE, "libgbmoe.so")
 
 # status codes, dtypes, scoring and FFN routes (values of include/gbmoe.h)
 OK, EINVAL, EUNSUPPORTED, EWORKSPACE, ECUDA, EDEVICE_TIMEOUT = 0, -1, -2, -3, -4, -5
-F32, BF16, FP8_E4M3_B128, INT4_G128 = 0, 1, 2, 3
+F32, BF16, FP8_E4M3_B128, INT4_G128, MXFP4 = 0, 1, 2, 3, 4
 SOFTMAX, SIGMOID = 0, 1
 FFN_AUTO, FFN_STREAM, FFN_SIMT, FFN_TC, FFN_TC_DEQUANT = 0, 1, 2, 3, 4
 
-DTYPES = {"f32": F32, "bf16": BF16, "fp8_b128": FP8_E4M3_B128, "int4_g128": INT4_G128}
+DTYPES = {"f32": F32, "bf16": BF16, "fp8_b128": FP8_E4M3_B128, "int4_g128": INT4_G128, "mxfp4": MXFP4}
 ROUTES = {"auto": FFN_AUTO, "stream": FFN_STREAM, "simt": FFN_SIMT, "tc": FFN_TC, "tc_dequant": FFN_TC_DEQUANT}
 
 # every function include/gbmoe.h declares

@@ -19,6 +19,8 @@ size_t align_up(size_t v) { return (v + kAlign - 1) & ~(kAlign - 1); }
 
 size_t act_bytes(int act) { return act == GBMOE_F32 ? 4 : 2; }
 
+bool quantised_weights(int w) { return w == GBMOE_FP8_E4M3_B128 || w == GBMOE_INT4_G128 || w == GBMOE_MXFP4; }
+
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
 int check_cfg(const gbmoe_config* c) {
@@ -27,7 +29,7 @@ int check_cfg(const gbmoe_config* c) {
     if (c->top_k > c->E) return GBMOE_EINVAL;
     if (c->score != GBMOE_SOFTMAX && c->score != GBMOE_SIGMOID) return GBMOE_EINVAL;
     if (c->act_dtype != GBMOE_F32 && c->act_dtype != GBMOE_BF16) return GBMOE_EINVAL;
-    if (c->w_dtype < GBMOE_F32 || c->w_dtype > GBMOE_INT4_G128) return GBMOE_EINVAL;
+    if (c->w_dtype < GBMOE_F32 || c->w_dtype > GBMOE_MXFP4) return GBMOE_EINVAL;
     if (c->has_shared != 0 && c->has_shared != 1) return GBMOE_EINVAL;
     if (c->has_shared && c->I_shared <= 0) return GBMOE_EINVAL;
     if (c->ffn_route < GBMOE_FFN_AUTO || c->ffn_route > GBMOE_FFN_TC_DEQUANT) return GBMOE_EINVAL;
@@ -65,8 +67,8 @@ int pick_route(const gbmoe_config* c, int64_t n_rows, int E, int I) {
         probe.I = I;
         probe.E = E;
         if (ffn_tc_supported(probe)) {
-            const bool quantised = c->w_dtype == GBMOE_FP8_E4M3_B128 || c->w_dtype == GBMOE_INT4_G128;
-            return quantised && n_rows >= kDequantRowsPerExpert * E ? GBMOE_FFN_TC_DEQUANT : GBMOE_FFN_TC;
+            return quantised_weights(c->w_dtype) && n_rows >= kDequantRowsPerExpert * E ? GBMOE_FFN_TC_DEQUANT
+                                                                                        : GBMOE_FFN_TC;
         }
     }
     return GBMOE_FFN_SIMT;
@@ -75,8 +77,7 @@ int pick_route(const gbmoe_config* c, int64_t n_rows, int E, int I) {
 // Bytes of the bf16 weight copy the TC_DEQUANT route decodes into (0 when
 // the route of that problem does not use one).
 size_t dequant_bytes(const gbmoe_config* c, int64_t n_rows, int E, int I) {
-    const bool quantised = c->w_dtype == GBMOE_FP8_E4M3_B128 || c->w_dtype == GBMOE_INT4_G128;
-    if (!quantised || pick_route(c, n_rows, E, I) != GBMOE_FFN_TC_DEQUANT) return 0;
+    if (!quantised_weights(c->w_dtype) || pick_route(c, n_rows, E, I) != GBMOE_FFN_TC_DEQUANT) return 0;
     return (size_t)3 * E * c->H * I * 2;
 }
 
@@ -131,9 +132,10 @@ int check_ws(const gbmoe_config* c, void* ws, size_t bytes) {
 int check_weights(const gbmoe_config* c, const gbmoe_expert_weights* w) {
     if (!w || !w->w_gate || !w->w_up || !w->w_down) return GBMOE_EINVAL;
     if (!aligned(w->w_gate, 16) || !aligned(w->w_up, 16) || !aligned(w->w_down, 16)) return GBMOE_EINVAL;
-    if (c->w_dtype == GBMOE_FP8_E4M3_B128 || c->w_dtype == GBMOE_INT4_G128) {
+    if (quantised_weights(c->w_dtype)) {
         if (!w->s_gate || !w->s_up || !w->s_down) return GBMOE_EINVAL;
-        if (!aligned(w->s_gate, 4) || !aligned(w->s_up, 4) || !aligned(w->s_down, 4)) return GBMOE_EINVAL;
+        const size_t sa = c->w_dtype == GBMOE_MXFP4 ? 2 : 4;  // E8M0 bytes are read in pairs
+        if (!aligned(w->s_gate, sa) || !aligned(w->s_up, sa) || !aligned(w->s_down, sa)) return GBMOE_EINVAL;
     }
     return GBMOE_OK;
 }

@@ -179,6 +179,21 @@ __device__ __forceinline__ float2 e4m3x2_to_f32x2(uint32_t two_bytes) {
 // signed 4-bit value of nibble n (two's complement)
 __device__ __forceinline__ float int4_to_f32(uint32_t n) { return (float)((int32_t)(n << 28) >> 28); }
 
+// FP4 E2M1 code (sign in bit 3, exponent bits 2-1 with bias 1, mantissa bit
+// 0) -> fp32, exact: the exponent and mantissa bits land in the fp32
+// exponent field 0..3 and the top mantissa bit, which reads as the value
+// times 2^-126 (the E2M1 subnormal 0.5 as the fp32 subnormal 2^-127), then
+// one multiply by 2^126.
+__device__ __forceinline__ float e2m1_to_f32(uint32_t c) {
+    const float v = __uint_as_float(((c & 8u) << 28) | ((c & 7u) << 22));
+    return v * __uint_as_float(0x7e800000u);  // 2^126
+}
+
+// E8M0 scale byte s -> 2^(s - 127) (s = 0: the fp32 subnormal 2^-127; 255: NaN)
+__device__ __forceinline__ float e8m0_to_f32(uint32_t s) {
+    return s == 255u ? __uint_as_float(0x7fc00000u) : s ? __uint_as_float(s << 23) : __uint_as_float(0x00400000u);
+}
+
 // ------------------------------------------------------------- silu
 
 __device__ __forceinline__ float silu_mul(float g, float u) { return g / (1.0f + expf(-g)) * u; }

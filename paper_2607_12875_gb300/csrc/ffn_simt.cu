@@ -141,6 +141,7 @@ cudaError_t launch_ffn_simt(const FfnProblem& p, cudaStream_t stream) {
             case GBMOE_BF16: return launch_simt_t<__nv_bfloat16, GBMOE_BF16>(p, stream);
             case GBMOE_FP8_E4M3_B128: return launch_simt_t<__nv_bfloat16, GBMOE_FP8_E4M3_B128>(p, stream);
             case GBMOE_INT4_G128: return launch_simt_t<__nv_bfloat16, GBMOE_INT4_G128>(p, stream);
+            case GBMOE_MXFP4: return launch_simt_t<__nv_bfloat16, GBMOE_MXFP4>(p, stream);
             default: return cudaErrorInvalidValue;
         }
     }
@@ -149,6 +150,7 @@ cudaError_t launch_ffn_simt(const FfnProblem& p, cudaStream_t stream) {
         case GBMOE_BF16: return launch_simt_t<float, GBMOE_BF16>(p, stream);
         case GBMOE_FP8_E4M3_B128: return launch_simt_t<float, GBMOE_FP8_E4M3_B128>(p, stream);
         case GBMOE_INT4_G128: return launch_simt_t<float, GBMOE_INT4_G128>(p, stream);
+        case GBMOE_MXFP4: return launch_simt_t<float, GBMOE_MXFP4>(p, stream);
         default: return cudaErrorInvalidValue;
     }
 }

@@ -19,6 +19,7 @@ cudaError_t launch_ffn_stream(const FfnProblem& p, cudaStream_t stream) {
         case GBMOE_BF16: return launch_stream_w<GBMOE_BF16>(p, stream);
         case GBMOE_FP8_E4M3_B128: return launch_stream_w<GBMOE_FP8_E4M3_B128>(p, stream);
         case GBMOE_INT4_G128: return launch_stream_w<GBMOE_INT4_G128>(p, stream);
+        case GBMOE_MXFP4: return launch_stream_w<GBMOE_MXFP4>(p, stream);
         default: return cudaErrorInvalidValue;
     }
 }

@@ -21,7 +21,8 @@
 //             y for the down GEMM; each warp stages 32 rows x 32 columns in
 //             shared memory and writes them with one TMA store.
 // Quantised weights (fp8 e4m3 with 128x128 block scales, int4 with 128-wide
-// group scales) take the same path with eight more warps: TMA brings the raw
+// group scales, MXFP4 with 32-wide E8M0 scales) take the same path with eight
+// more warps: TMA brings the raw
 // weight tile (64- or 32-byte swizzled rows) next to the A tile, and
 // warps 6-13, one B row per thread, decode it, apply the scale and write
 // the bf16 operand in the 128-byte-swizzled layout the MMA reads, then
@@ -69,6 +70,14 @@ template <>
 struct Fmt<GBMOE_INT4_G128> {
     static constexpr int RAW_BYTES = BN * BK / 2, STAGES = 4, THREADS = 192 + CONVERT_WARPS * 32;
 };
+template <>
+struct Fmt<GBMOE_MXFP4> {
+    static constexpr int RAW_BYTES = BN * BK / 2, STAGES = 4, THREADS = 192 + CONVERT_WARPS * 32;
+};
+
+// nibble-packed formats: a raw row of BK elements is BK / 2 bytes
+template <int WQ>
+constexpr bool packed4() { return WQ == GBMOE_INT4_G128 || WQ == GBMOE_MXFP4; }
 
 template <int WQ>
 struct Layout {
@@ -324,6 +333,35 @@ __device__ __forceinline__ uint4 decode_int4_8(uint32_t w, __nv_bfloat162 sc2) {
                       __byte_perm(p[0], p[1], 0x7632), __byte_perm(p[2], p[3], 0x7632));
 }
 
+// 8 FP4 E2M1 weights (one 32-bit word, element 0 in the low nibble) times the
+// E8M0 block scale (sc2 = 2^(s-127) in both halves) -> 8 bf16 (one 16-byte
+// chunk), exact. A code's exponent and mantissa bits are placed in the bf16
+// exponent field 0..3 and top mantissa bit, which reads as the value times
+// 2^-126 (the E2M1 subnormal 0.5 as the bf16 subnormal 2^-127); one bf16
+// multiply by 2^126 and one by the scale, both exact.
+__device__ __forceinline__ uint4 decode_mxfp4_8(uint32_t w, __nv_bfloat162 sc2) {
+    const uint32_t k2p126 = 0x7e807e80u;  // bf16x2 (2^126, 2^126)
+    uint32_t p[4];  // p[i] holds elements (i, i + 4)
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const uint32_t t = (w >> (4 * i)) & 0x000f000fu;
+        uint32_t b = ((t & 0x00080008u) << 12) | ((t & 0x00070007u) << 6);
+        __nv_bfloat162 v = __hmul2(*reinterpret_cast<__nv_bfloat162*>(&b),
+                                   *reinterpret_cast<const __nv_bfloat162*>(&k2p126));
+        v = __hmul2(v, sc2);
+        p[i] = *reinterpret_cast<uint32_t*>(&v);
+    }
+    return make_uint4(__byte_perm(p[0], p[1], 0x5410), __byte_perm(p[2], p[3], 0x5410),
+                      __byte_perm(p[0], p[1], 0x7632), __byte_perm(p[2], p[3], 0x7632));
+}
+
+// E8M0 byte -> bf16x2 (2^(s-127), 2^(s-127)); s = 0 is the bf16 subnormal 2^-127
+__device__ __forceinline__ __nv_bfloat162 e8m0_bf16x2(uint32_t s) {
+    const uint32_t h = s ? (s << 7) : 0x0040u;
+    const uint32_t b = h | (h << 16);
+    return *reinterpret_cast<const __nv_bfloat162*>(&b);
+}
+
 // ------------------------------------------------------------------ kernel
 
 struct Work {
@@ -433,7 +471,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
                     tma_load_2d(sB + stage * B_BYTES + B_BYTES / 2, &tm_b1, kb * BK, b1, &full[stage]);
                 } else {
                     // raw boxes are BK elements wide: BK bytes (fp8) or BK/2 bytes (int4)
-                    const int x = (WQ == GBMOE_INT4_G128) ? kb * (BK / 2) : kb * BK;
+                    const int x = packed4<WQ>() ? kb * (BK / 2) : kb * BK;
                     tma_load_2d(sR + stage * RAW, &tm_b0, x, b0, &full[stage]);
                     tma_load_2d(sR + stage * RAW + RAW / 2, &tm_b1, x, b1, &full[stage]);
                 }
@@ -546,19 +584,24 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
             int b0, b1;
             b_rows(p, wk, b0, b1);
             const int64_t brow = (half ? b1 : b0) + (r & 127);  // absolute row of the stacked B tensor
-            // scale of this row for 128-wide k group j: one per 128x128 block (fp8)
-            // or per row (int4), loaded four groups ahead so that no k-block waits
-            // on a global load before decoding
+            // scale entry j of this row, loaded four entries ahead so that no
+            // k-block waits on a global load before decoding: for the 128-wide
+            // k group j one fp32 per 128x128 block (fp8) or one bf16 per row
+            // (int4); for MXFP4 the two E8M0 bytes of k-block j (as raw bits)
+            constexpr int KB_PER_SCALE = WQ == GBMOE_MXFP4 ? 1 : 2;
             auto scale_of = [&](int j) -> float {
-                if (j >= kgroups) return 0.0f;
+                if (j >= nkb / KB_PER_SCALE) return 0.0f;
                 if (WQ == GBMOE_FP8_E4M3_B128) return static_cast<const float*>(scales)[(brow / 128) * kgroups + j];
+                if (WQ == GBMOE_MXFP4)
+                    return __uint_as_float(
+                        *reinterpret_cast<const uint16_t*>(static_cast<const uint8_t*>(scales) + brow * (p.K / 32) + 2 * j));
                 return __bfloat162float(static_cast<const __nv_bfloat16*>(scales)[brow * kgroups + j]);
             };
             float sc0 = scale_of(0), sc1 = scale_of(1), sc2 = scale_of(2), sc3 = scale_of(3);
             for (int kb = 0; kb < nkb; ++kb) {
-                if (kb > 0 && (kb & 1) == 0) {  // next 128-wide group
+                if (kb > 0 && kb % KB_PER_SCALE == 0) {  // next scale entry
                     sc0 = sc1; sc1 = sc2; sc2 = sc3;
-                    sc3 = scale_of(kb / 2 + 3);
+                    sc3 = scale_of(kb / KB_PER_SCALE + 3);
                 }
                 if (!warp_wait(&full[stage], phase, abort_flag, p.err, p.wait_limit_ns)) { ok = false; break; }
                 const uint8_t* raw = sR + stage * RAW;
@@ -571,6 +614,17 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
                         decode_fp8_16(v, sc0, o0, o1);
                         *reinterpret_cast<uint4*>(dstB + sw128_off(r, 2 * c)) = o0;
                         *reinterpret_cast<uint4*>(dstB + sw128_off(r, 2 * c + 1)) = o1;
+                    }
+                } else if (WQ == GBMOE_MXFP4) {
+                    const uint32_t pair = __float_as_uint(sc0);  // E8M0 of elements 0-31, 32-63
+#pragma unroll
+                    for (int c = 0; c < 2; ++c) {
+                        const __nv_bfloat162 scv = e8m0_bf16x2((pair >> (8 * c)) & 0xffu);
+                        const uint4 v = *reinterpret_cast<const uint4*>(raw + sw32_off(r, c));
+                        const uint32_t ws[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+                        for (int i = 0; i < 4; ++i)
+                            *reinterpret_cast<uint4*>(dstB + sw128_off(r, 4 * c + i)) = decode_mxfp4_8(ws[i], scv);
                     }
                 } else {
                     const __nv_bfloat162 sc2v = __float2bfloat162_rn(sc0);  // exact: sc0 came from a bf16
@@ -645,7 +699,9 @@ dequant_weights_kernel(const uint8_t* __restrict__ w, const void* __restrict__ s
         uint4* dst = reinterpret_cast<uint4*>(out + row * K);
         // scale of 128-wide k group g of this row
         const float* s8 = kFp8 ? static_cast<const float*>(s) + (e * (N / 128) + n / 128) * kgroups : nullptr;
-        const __nv_bfloat16* s4 = kFp8 ? nullptr : static_cast<const __nv_bfloat16*>(s) + row * kgroups;
+        const __nv_bfloat16* s4 =
+            WQ == GBMOE_INT4_G128 ? static_cast<const __nv_bfloat16*>(s) + row * kgroups : nullptr;
+        const uint8_t* smx = WQ == GBMOE_MXFP4 ? static_cast<const uint8_t*>(s) + row * (K / 32) : nullptr;
         for (int p0 = lane; p0 < ppr; p0 += 32 * kDqUnroll) {
             uint2 raw[kDqUnroll];
 #pragma unroll
@@ -666,6 +722,8 @@ dequant_weights_kernel(const uint8_t* __restrict__ w, const void* __restrict__ s
                     uint4 o0, o1;  // decode_fp8_16 takes 16 bytes; the upper 8 are unused here
                     decode_fp8_16(make_uint4(raw[u].x, raw[u].y, 0, 0), s8[g], o0, o1);
                     dst[pc] = o0;
+                } else if constexpr (WQ == GBMOE_MXFP4) {
+                    dst[pc] = decode_mxfp4_8(raw[u].x, e8m0_bf16x2(smx[pc >> 2]));  // 4 pieces per 32-block
                 } else {
                     dst[pc] = decode_int4_8(raw[u].x, __float2bfloat162_rn(__bfloat162float(s4[g])));
                 }
@@ -725,6 +783,7 @@ static bool map_weights(CUtensorMap* m, int wq, const void* base, int64_t rows, 
         case GBMOE_FP8_E4M3_B128:
             return make_map(m, base, rows, K, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, BK, CU_TENSOR_MAP_SWIZZLE_64B);
         case GBMOE_INT4_G128:
+        case GBMOE_MXFP4:
             return make_map(m, base, rows, K / 2, CU_TENSOR_MAP_DATA_TYPE_UINT8, 1, BK / 2, CU_TENSOR_MAP_SWIZZLE_32B);
         default: return false;
     }
@@ -754,6 +813,7 @@ static cudaError_t launch_gemm(int wq, const CUtensorMap& a, const CUtensorMap& 
         case GBMOE_FP8_E4M3_B128:
             return launch_gemm_t<GBMOE_FP8_E4M3_B128>(a, b0, b1, out, prm, max_work, stream);
         case GBMOE_INT4_G128: return launch_gemm_t<GBMOE_INT4_G128>(a, b0, b1, out, prm, max_work, stream);
+        case GBMOE_MXFP4: return launch_gemm_t<GBMOE_MXFP4>(a, b0, b1, out, prm, max_work, stream);
         default: return cudaErrorInvalidValue;
     }
 }
@@ -761,7 +821,8 @@ static cudaError_t launch_gemm(int wq, const CUtensorMap& a, const CUtensorMap& 
 }  // namespace tc
 
 bool ffn_tc_supported(const FfnProblem& p) {
-    const bool wq_ok = p.w_dtype == GBMOE_BF16 || p.w_dtype == GBMOE_FP8_E4M3_B128 || p.w_dtype == GBMOE_INT4_G128;
+    const bool wq_ok = p.w_dtype == GBMOE_BF16 || p.w_dtype == GBMOE_FP8_E4M3_B128 ||
+                       p.w_dtype == GBMOE_INT4_G128 || p.w_dtype == GBMOE_MXFP4;
     return p.act_dtype == GBMOE_BF16 && wq_ok && p.H % 256 == 0 && p.I % 128 == 0 && tc::encode_fn() != nullptr;
 }
 
@@ -777,12 +838,11 @@ static cudaError_t dequant_all(const FfnProblem& p, FfnProblem& q, cudaStream_t 
                            {p.w_down, p.s_down, p.H, p.I, dq + 2 * gu}};
     for (const Part& pt : parts) {
         const dim3 grid((unsigned)((pt.N + kDqWarps - 1) / kDqWarps), (unsigned)p.E);
-        const cudaError_t err =
-            p.w_dtype == GBMOE_FP8_E4M3_B128
-                ? launch_k(dequant_weights_kernel<GBMOE_FP8_E4M3_B128>, dim3(grid), dim3(kDqWarps * 32), 0, stream,
-                           static_cast<const uint8_t*>(pt.w), pt.s, pt.N, pt.K, p.sched, pt.out)
-                : launch_k(dequant_weights_kernel<GBMOE_INT4_G128>, dim3(grid), dim3(kDqWarps * 32), 0, stream,
-                           static_cast<const uint8_t*>(pt.w), pt.s, pt.N, pt.K, p.sched, pt.out);
+        auto kernel = p.w_dtype == GBMOE_FP8_E4M3_B128 ? dequant_weights_kernel<GBMOE_FP8_E4M3_B128>
+                      : p.w_dtype == GBMOE_MXFP4        ? dequant_weights_kernel<GBMOE_MXFP4>
+                                                        : dequant_weights_kernel<GBMOE_INT4_G128>;
+        const cudaError_t err = launch_k(kernel, dim3(grid), dim3(kDqWarps * 32), 0, stream,
+                                         static_cast<const uint8_t*>(pt.w), pt.s, pt.N, pt.K, p.sched, pt.out);
         if (err != cudaSuccess) return err;
     }
     q.w_dtype = GBMOE_BF16;
@@ -810,7 +870,8 @@ cudaError_t launch_ffn_tc(const FfnProblem& pin, cudaStream_t stream) {
     cudaError_t err = launch_ffn_schedule(pin.counts, pin.E, pin.n_rows, BM, pin.sched, stream);
     if (err != cudaSuccess) return err;
     FfnProblem p = pin;
-    if (pin.w_dq && (pin.w_dtype == GBMOE_FP8_E4M3_B128 || pin.w_dtype == GBMOE_INT4_G128))
+    if (pin.w_dq && (pin.w_dtype == GBMOE_FP8_E4M3_B128 || pin.w_dtype == GBMOE_INT4_G128 ||
+                     pin.w_dtype == GBMOE_MXFP4))
         if ((err = dequant_all(pin, p, stream)) != cudaSuccess) return err;
     // A operand of the gate/up GEMM: x rows in sorted order (a gathered copy),
     // or x itself when rows are already in order (no sorted_pair: shared expert)

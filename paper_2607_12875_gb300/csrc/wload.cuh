@@ -2,6 +2,7 @@
 //   F32 / BF16       plain values
 //   FP8_E4M3_B128    e4m3 bytes, fp32 scale per 128x128 block of the [N, K] matrix
 //   INT4_G128        two's complement nibbles (even k low), bf16 scale per 128 k of a row
+//   MXFP4            E2M1 nibbles (even k low), E8M0 scale per 32 k of a row
 #pragma once
 
 #include "common.cuh"
@@ -96,6 +97,32 @@ struct WFmt<GBMOE_INT4_G128> {
         uint32_t b = static_cast<const uint8_t*>(w)[((size_t)e * N + n) * (K / 2) + k / 2];
         uint32_t nib = (k & 1) ? (b >> 4) : (b & 0xfu);
         return int4_to_f32(nib) * scale(s, e, N, K, n, k);
+    }
+};
+
+template <>
+struct WFmt<GBMOE_MXFP4> {
+    static constexpr int CE = 32;  // one 16-byte chunk = one 32-element scale block
+    static constexpr int NV = 1;
+    __device__ static size_t row_bytes(int K) { return (size_t)K / 2; }
+    __device__ static float scale(const void* s, int64_t e, int N, int K, int n, int k) {
+        return e8m0_to_f32(static_cast<const uint8_t*>(s)[((size_t)e * N + n) * (K / 32) + k / 32]);
+    }
+    __device__ static const void* scale_row(const void* s, int64_t e, int N, int K, int n) {
+        return static_cast<const uint8_t*>(s) + ((size_t)e * N + n) * (K / 32);
+    }
+    __device__ static float scale_at(const void* row, int k) {
+        return e8m0_to_f32(static_cast<const uint8_t*>(row)[k / 32]);
+    }
+    __device__ __forceinline__ static void decode8(const uint4 (&r)[NV], int sub, float sc, float (&w)[8]) {
+        uint32_t v = sub == 0 ? r[0].x : sub == 1 ? r[0].y : sub == 2 ? r[0].z : r[0].w;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) w[i] = e2m1_to_f32((v >> (4 * i)) & 0xfu) * sc;
+    }
+    __device__ static float elem(const void* w, const void* s, int64_t e, int N, int K, int n, int k) {
+        uint32_t b = static_cast<const uint8_t*>(w)[((size_t)e * N + n) * (K / 2) + k / 2];
+        uint32_t nib = (k & 1) ? (b >> 4) : (b & 0xfu);
+        return e2m1_to_f32(nib) * scale(s, e, N, K, n, k);
     }
 };
 

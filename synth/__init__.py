@@ -45,6 +45,7 @@ def _L():
         lib.synth_normal_bf16.argtypes = [u64, u64, dbl, u64, i64, vp]
         lib.synth_fp8_b128.argtypes = [u64, u64, dbl, i64, i64, i64, i64, vp, vp]
         lib.synth_int4_g128.argtypes = [u64, u64, dbl, i64, i64, i64, i64, vp, vp]
+        lib.synth_mxfp4.argtypes = [u64, u64, dbl, i64, i64, i64, i64, vp, vp]
         lib.synth_set_threads.argtypes = [ctypes.c_int]
         lib.synth_set_threads(os.cpu_count() or 1)
         _lib = lib
@@ -89,6 +90,16 @@ def int4_g128(seed, tid, sigma, N, K, e0=0, ne=1):
     return q, s
 
 
+def mxfp4(seed, tid, sigma, N, K, e0=0, ne=1):
+    """Experts [e0, e0+ne) of an [E, N, K] weight as MXFP4 (packed E2M1
+    [ne, N, K/2] u8, E8M0 block scales [ne, N, K/32] u8)."""
+    q = np.empty((ne, N, K // 2), dtype=np.uint8)
+    s = np.empty((ne, N, K // 32), dtype=np.uint8)
+    if _L().synth_mxfp4(seed, tid, sigma, e0, ne, N, K, _ptr(q), _ptr(s)) != 0:
+        raise ValueError("MXFP4 blocks of 32 need K to be a multiple of 32")
+    return q, s
+
+
 def bf16_bits_to_f32(b: np.ndarray) -> np.ndarray:
     """Exact widening of raw bf16 bit patterns to fp32."""
     return (b.astype(np.uint32) << 16).view(np.float32)
@@ -105,7 +116,7 @@ class Workload:
     E: int
     top_k: int
     act: str            # "f32" | "bf16"   (x, router weight, h, y, out)
-    wq: str             # "f32" | "bf16" | "fp8_b128" | "int4_g128"  (expert weights)
+    wq: str             # "f32" | "bf16" | "fp8_b128" | "int4_g128" | "mxfp4"  (expert weights)
     seed: int
     score: str = "softmax"      # "softmax" | "sigmoid"
     renormalize: bool = True
@@ -138,6 +149,11 @@ WORKLOADS = {
                 has_shared=True, I_shared=2048, select_bias_sigma=0.01),
     5: Workload("skew_int4_T16384_H4096_E64_k6_I2816", 16384, 4096, 2816, 64, 6, "bf16", "int4_g128",
                 seed=4, zipf=True),
+    # the DeepSeek-style layer of workload 4 with MXFP4 expert weights (the
+    # expert format of the DeepSeek reference path, Section 6.2)
+    6: Workload("dsv4_mxfp4_T2048_H7168_E256s1_k8_I2048", 2048, 7168, 2048, 256, 8, "bf16", "mxfp4",
+                seed=5, score="sigmoid", routed_scale=2.5, n_group=8, topk_group=4,
+                has_shared=True, I_shared=2048, select_bias_sigma=0.01),
 }
 
 
@@ -174,6 +190,9 @@ def expert_weights(w: Workload, E: int, I: int, tids=("w_gate", "w_up", "w_down"
             out["w_" + name], out["s_" + name] = q, s
         elif w.wq == "int4_g128":
             q, s = int4_g128(w.seed, TID[tid], w.w_sigma, N, K, e0, ne)
+            out["w_" + name], out["s_" + name] = q, s
+        elif w.wq == "mxfp4":
+            q, s = mxfp4(w.seed, TID[tid], w.w_sigma, N, K, e0, ne)
             out["w_" + name], out["s_" + name] = q, s
         else:
             raise ValueError(w.wq)

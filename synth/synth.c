@@ -23,6 +23,11 @@
  *   int4 symmetric, groups of 128 along K: s = bf16(amax(group) / 7),
  *     q = clamp(rne(w / s), -8, 7); two's complement nibbles, the even k in
  *     the low nibble; s = 1 if amax = 0.
+ *   MXFP4 (OCP Microscaling Formats v1.0), blocks of 32 along K: shared
+ *     scale X = 2^(floor(log2(amax)) - 2) stored as its E8M0 exponent
+ *     (biased by 127; 2 is the largest exponent of FP4 E2M1), elements
+ *     q = E2M1(w / X) rounded to nearest, ties to an even code, saturating
+ *     at +-6; sign in bit 3, even k in the low nibble; X = 1 if amax = 0.
  */
 #include <math.h>
 #include <pthread.h>
@@ -255,5 +260,70 @@ int synth_int4_g128(uint64_t seed, uint64_t tensor_id, double sigma, int64_t e0,
     if (K % 128) return -1;
     int4_ctx c = {synth_stream_key(seed, tensor_id), sigma_scale(sigma), N, K, e0, q, s};
     parallel_for(ne * N * (K / 128), int4_range, &c);
+    return 0;
+}
+
+/* ------------------------------------- MXFP4: E2M1 + E8M0 per 32 along K */
+
+/* Magnitude code (0..7) of FP4 E2M1 nearest to a >= 0, ties to the even
+ * code, saturating at 6. Grid: 0, 0.5, 1, 1.5, 2, 3, 4, 6. */
+static int e2m1_code(double a) {
+    static const double grid[8] = {0.0, 0.5, 1.0, 1.5, 2.0, 3.0, 4.0, 6.0};
+    if (a >= 6.0) return 7;
+    int best = 0;
+    for (int c = 1; c < 8; ++c) {
+        double d = fabs(a - grid[c]), db = fabs(a - grid[best]);
+        if (d < db || (d == db && (c & 1) == 0)) best = c;
+    }
+    return best;
+}
+
+typedef struct {
+    uint64_t key; float scale; int64_t N, K; int64_t e0;
+    uint8_t* q; uint8_t* s;
+} mxfp4_ctx;
+
+static void mxfp4_range(void* p, int64_t b, int64_t e) {
+    mxfp4_ctx* c = (mxfp4_ctx*)p;
+    const int64_t kg = c->K / 32;
+    float g[32];
+    for (int64_t blk = b; blk < e; ++blk) {
+        int64_t row = blk / kg, gk = blk % kg; /* row = ex * N + n */
+        int64_t ex = row / c->N, n = row % c->N;
+        float amax = 0.0f;
+        for (int j = 0; j < 32; ++j) {
+            uint64_t idx = (uint64_t)(((c->e0 + ex) * c->N + n) * c->K + gk * 32 + j);
+            g[j] = normal_f32(c->key, idx, c->scale);
+            float av = fabsf(g[j]);
+            if (av > amax) amax = av;
+        }
+        int ex2 = 0; /* scale exponent: floor(log2(amax)) - 2 */
+        if (amax > 0.0f) {
+            int fe;
+            frexp((double)amax, &fe); /* amax in [2^(fe-1), 2^fe) */
+            ex2 = (fe - 1) - 2;
+        }
+        int biased = ex2 + 127;
+        if (biased < 0) biased = 0;
+        if (biased > 254) biased = 254;
+        c->s[blk] = (uint8_t)biased;
+        const double X = ldexp(1.0, biased - 127);
+        uint8_t* dst = c->q + row * (c->K / 2) + gk * 16;
+        for (int j = 0; j < 32; j += 2) {
+            int n0 = e2m1_code(fabs((double)g[j]) / X) | (g[j] < 0.0f ? 8 : 0);
+            int n1 = e2m1_code(fabs((double)g[j + 1]) / X) | (g[j + 1] < 0.0f ? 8 : 0);
+            dst[j / 2] = (uint8_t)(n0 | (n1 << 4));
+        }
+    }
+}
+
+/* Experts [e0, e0+ne) of a [E, N, K] weight drawn from N(0, sigma^2) and stored
+ * as MXFP4: packed E2M1 q [ne, N, K/2] (even k in the low nibble) with E8M0
+ * block scales s [ne, N, K/32]. Returns -1 unless K is a multiple of 32. */
+int synth_mxfp4(uint64_t seed, uint64_t tensor_id, double sigma, int64_t e0, int64_t ne, int64_t N,
+                int64_t K, uint8_t* q, uint8_t* s) {
+    if (K % 32) return -1;
+    mxfp4_ctx c = {synth_stream_key(seed, tensor_id), sigma_scale(sigma), N, K, e0, q, s};
+    parallel_for(ne * N * (K / 32), mxfp4_range, &c);
     return 0;
 }

@@ -8,12 +8,14 @@ import torch
 import paper_2607_12875_gb300 as gb
 import synth
 
-TOL = {"f32": 1e-5, "bf16": 2e-2, "fp8_b128": 5e-2, "int4_g128": 5e-2}
+TOL = {"f32": 1e-5, "bf16": 2e-2, "fp8_b128": 5e-2, "int4_g128": 5e-2, "mxfp4": 2e-2}
 
 
 def tol_for(wl) -> float:
-    """Output tolerance of a workload: 1e-5 for fp32, 2e-2 for bf16, 5e-2 for fp8/int4 weights."""
-    if wl.wq in ("fp8_b128", "int4_g128"):
+    """Output tolerance of a workload: 1e-5 for fp32, 2e-2 for bf16, 5e-2 for
+    fp8/int4 weights; MXFP4 weights decode exactly (to bf16 and fp32), so they
+    take the bf16 bound."""
+    if wl.wq in ("fp8_b128", "int4_g128", "mxfp4"):
         return TOL[wl.wq]
     return TOL["f32"] if wl.act == "f32" and wl.wq == "f32" else TOL["bf16"]
 
@@ -34,8 +36,8 @@ def dev_weights(store: dict, wq: str, device="cuda") -> dict:
                 out[k] = torch.from_numpy(v.view(np.int16)).to(device).view(torch.bfloat16)
             else:
                 out[k] = torch.from_numpy(v).to(device)
-        else:  # scales
-            if wq == "fp8_b128":
+        else:  # scales: fp32 (fp8), E8M0 bytes (MXFP4), bf16 bits (int4)
+            if wq in ("fp8_b128", "mxfp4"):
                 out[k] = torch.from_numpy(v).to(device)
             else:
                 out[k] = torch.from_numpy(v.view(np.int16)).to(device).view(torch.bfloat16)

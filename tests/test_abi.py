@@ -50,7 +50,7 @@ def cfg_of(wid, **kw):
     return c
 
 
-@pytest.mark.parametrize("wid", [1, 2, 3, 4, 5])
+@pytest.mark.parametrize("wid", [1, 2, 3, 4, 5, 6])
 def test_workload_configs_are_valid(lib, wid):
     c = cfg_of(wid)
     assert gb.check_config(c) == gb.OK
@@ -66,6 +66,7 @@ def test_workload_configs_are_valid(lib, wid):
     (dict(T=-1), gb.EINVAL),
     (dict(score=7), gb.EINVAL),
     (dict(act_dtype=2), gb.EINVAL),
+    (dict(w_dtype=5), gb.EINVAL),
     (dict(ffn_route=9), gb.EINVAL),
     (dict(ffn_route=gb.FFN_TC), gb.EUNSUPPORTED),  # fp32 activations have no tensor-core route
     (dict(ffn_route=gb.FFN_TC_DEQUANT), gb.EUNSUPPORTED),
@@ -129,7 +130,7 @@ def test_entry_points_reject_bad_arguments_before_launching(lib):
     assert gb.status_string(gb.EDEVICE_TIMEOUT) == "device-side wait timed out"
 
 
-@pytest.mark.parametrize("wid", [4, 5])
+@pytest.mark.parametrize("wid", [4, 5, 6])
 def test_dequant_route_workspace_holds_bf16_weight_copies(lib, wid):
     """Forcing the decode-once route adds one bf16 copy of every expert's
     gate, up and down matrices (and of the shared expert's) to the workspace."""

@@ -11,7 +11,7 @@ import bench  # noqa: E402
 import synth  # noqa: E402
 
 
-@pytest.mark.parametrize("wq", ["f32", "bf16", "fp8_b128", "int4_g128"])
+@pytest.mark.parametrize("wq", ["f32", "bf16", "fp8_b128", "int4_g128", "mxfp4"])
 @pytest.mark.parametrize("H,I", [(256, 128), (512, 384)])
 def test_expert_bytes_match_generated_arrays(wq, H, I):
     wl = synth.WORKLOADS[1].replace(H=H, I=I, E=2, top_k=1, wq=wq, act="f32" if wq == "f32" else "bf16")

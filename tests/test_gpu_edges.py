@@ -79,7 +79,7 @@ def test_k_equals_E_and_single_expert(route):
     check(TINY.replace(T=9, E=1, top_k=1, seed=25), route)
 
 
-@pytest.mark.parametrize("wq", ["fp8_b128", "int4_g128"])
+@pytest.mark.parametrize("wq", ["fp8_b128", "int4_g128", "mxfp4"])
 @pytest.mark.parametrize("route", ["simt", "stream"])
 def test_quantised_weights_small(wq, route):
     wl = TINY.replace(T=24, E=4, top_k=2, act="bf16", wq=wq, H=256, I=256, seed=26)
@@ -164,3 +164,14 @@ def test_maximum_experts_and_top_k(score, act, route):
     assert gb.check_config(config(wl, route)) == gb.OK
     ref = check(wl, route)
     assert (ref["counts"] > 0).sum() > 200
+
+
+@pytest.mark.parametrize("route", ["simt", "stream"])
+def test_mxfp4_with_fp32_activations(route):
+    """MXFP4 weights under fp32 activations (the exact-decode format on the
+    fp32 routes, held to the fp32 bound of 1e-5)."""
+    wl = TINY.replace(T=30, E=4, top_k=2, act="f32", wq="mxfp4", H=256, I=256, seed=28)
+    inp, out, ids, counts = run(wl, route)
+    ref = oracle.forward(wl, inp)
+    assert np.array_equal(ids.cpu().numpy(), ref["topk_ids"])
+    assert_close(act_np(out), ref["out"], 1e-5)

@@ -1,5 +1,6 @@
 """GPU parity: every C-ABI call of the layer against the CPU oracle on the
-same seeded inputs, for all five workload shapes and every FFN route.
+same seeded inputs, for the five workload shapes, the MXFP4 variant of the
+DeepSeek-style layer (workload 6), and every FFN route.
 Routing ids, the permutation and the counts must match bit for bit; outputs
 within the workload's tolerance, as the infinity-norm relative error
 max |gpu - oracle| / max |oracle| and as every row's relative error (floored,
@@ -18,11 +19,11 @@ from gpu_helpers import (act_np, assert_close, config, rel_err, tiles_covered, t
 pytestmark = pytest.mark.gpu
 
 ROUTES = {1: ["simt", "stream", "auto"], 2: ["stream", "simt", "auto"], 3: ["simt", "auto"],
-          4: ["simt", "auto", "tc_dequant"], 5: ["simt", "auto", "tc"]}
+          4: ["simt", "auto", "tc_dequant"], 5: ["simt", "auto", "tc"], 6: ["simt", "auto", "tc_dequant"]}
 ALL_ROUTES = ["auto", "stream", "simt", "tc", "tc_dequant"]
 
 
-@pytest.fixture(scope="module", params=[1, 2, 3, 4, 5])
+@pytest.fixture(scope="module", params=[1, 2, 3, 4, 5, 6])
 def wcase(request):
     """Host inputs, device inputs and the full oracle forward of one workload.
     Module scope with parameters: pytest runs all tests of one workload

@@ -29,7 +29,7 @@ def forward(wl, dev, route):
     return out, ids
 
 
-@pytest.mark.parametrize("wq", ["bf16", "fp8_b128", "int4_g128"])
+@pytest.mark.parametrize("wq", ["bf16", "fp8_b128", "int4_g128", "mxfp4"])
 @pytest.mark.parametrize("T,E,k,H,I", [(200, 4, 2, 512, 256), (1000, 4, 2, 256, 384), (333, 16, 3, 768, 128)])
 def test_tc_small_ragged(T, E, k, H, I, wq):
     wl = BASE.replace(T=T, E=E, top_k=k, H=H, I=I, seed=T + E, wq=wq)
@@ -52,7 +52,7 @@ def test_tc_sigmoid_grouped_fp8_with_shared_expert():
     assert_close(act_np(out), ref["out"], tol_for(wl))
 
 
-@pytest.mark.parametrize("wq", ["fp8_b128", "int4_g128"])
+@pytest.mark.parametrize("wq", ["fp8_b128", "int4_g128", "mxfp4"])
 @pytest.mark.parametrize("T,E,k,H,I", [(200, 4, 2, 512, 256), (333, 16, 3, 768, 128)])
 def test_dequant_route_equals_in_gemm_decode(T, E, k, H, I, wq):
     """Decoding the weights once into a bf16 copy gives the GEMM the same bf16
@@ -89,6 +89,8 @@ def test_auto_route_choice():
     assert gb.ffn_route(config(synth.WORKLOADS[4])) == "tc"
     assert gb.ffn_route(config(synth.WORKLOADS[4]), shared=True) == "tc_dequant"
     assert gb.ffn_route(config(synth.WORKLOADS[5])) == "tc_dequant"
+    assert gb.ffn_route(config(synth.WORKLOADS[6])) == "tc"
+    assert gb.ffn_route(config(synth.WORKLOADS[6]), shared=True) == "tc_dequant"
 
 
 @pytest.mark.parametrize("wq", ["bf16", "int4_g128"])
