@@ -387,6 +387,8 @@ def measure(args, wid: int, overrides, dist, world: int, rank: int, local: int, 
               "tc": "moe_grouped_ffn, tcgen05 route (row gather + gate/up GEMM with SwiGLU + down GEMM)",
               "tc_dequant": "moe_grouped_ffn, tcgen05 decode-once route (3 weight-decode passes + row gather + "
                             "gate/up GEMM with SwiGLU + down GEMM)",
+              "tc_fp8": "moe_grouped_ffn, fp8 tcgen05 route (two-term e4m3 quantisation of the rows + gate/up "
+                        "GEMM with per-k-block promotion and SwiGLU + quantisation of h + down GEMM)",
               "simt": "moe_grouped_ffn, CUDA-core route"}[route]
     tpe = TRAFFIC_PER_ACTIVE_EXPERT.get((wl.name, route))
     extra = {"traffic": None if tpe is None else tpe * active, "kernel": kernel, "active_experts": active,
@@ -434,7 +436,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", type=int, default=2, help="synth.WORKLOADS id of the headline (2 = decode bf16)")
-    ap.add_argument("--route", default="auto", choices=["auto", "stream", "simt", "tc", "tc_dequant"])
+    ap.add_argument("--route", default="auto", choices=["auto", "stream", "simt", "tc", "tc_dequant", "tc_fp8"])
     ap.add_argument("--ref-tokens", type=int, default=1, help="tokens per oracle step (reference arm)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-per-config", action="store_true",

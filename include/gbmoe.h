@@ -63,7 +63,15 @@ enum {
 /* Router scoring. */
 enum { GBMOE_SOFTMAX = 0, GBMOE_SIGMOID = 1 };
 
-/* Which expert-FFN kernels run. AUTO streams weights when the average number
+/* Which expert-FFN kernels run. GBMOE_FFN_TC_FP8 (FP8_E4M3_B128 weights and
+ * bf16 activations only) follows the DeepSeek-V3 recipe: each GEMM's input
+ * rows (x, then h) are quantised to e4m3 with one fp32 scale per row and 128
+ * consecutive k (scale = amax / 448, round to nearest even), the tensor cores
+ * multiply e4m3 by e4m3, and each 128-wide k block's partial sum is scaled by
+ * both blocks' scales and accumulated in fp32. The activation rounding makes
+ * its outputs differ from the other routes' by about 1-3% of their typical
+ * magnitude (the fp8 tolerance, 5e-2 of the largest output, covers it).
+ * AUTO streams weights when the average number
  * of rows per expert P/E is at most 16 and otherwise runs the grouped GEMM
  * (tensor cores for bf16 activations, CUDA cores for fp32). On the tensor
  * cores, fp8/int4/MXFP4 weights are decoded inside the GEMM when P/E < 256; with
@@ -76,7 +84,9 @@ enum {
     GBMOE_FFN_STREAM = 1,     /* weight streaming: few rows per expert (decode)       */
     GBMOE_FFN_SIMT = 2,       /* CUDA-core tiled GEMM (fp32 activations, any weights) */
     GBMOE_FFN_TC = 3,         /* tcgen05/TMEM/TMA grouped GEMM (bf16 activations)     */
-    GBMOE_FFN_TC_DEQUANT = 4  /* as TC, quantised weights decoded once beforehand     */
+    GBMOE_FFN_TC_DEQUANT = 4, /* as TC, quantised weights decoded once beforehand     */
+    GBMOE_FFN_TC_FP8 = 5      /* fp8 tensor cores: FP8_E4M3_B128 weights as stored,
+                                 activations quantised to e4m3 per 1x128 block      */
 };
 
 typedef struct gbmoe_config {

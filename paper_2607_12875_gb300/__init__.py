@@ -19,10 +19,11 @@ LIB_PATH = os.path.join(_HERE, "libgbmoe.so")
 OK, EINVAL, EUNSUPPORTED, EWORKSPACE, ECUDA, EDEVICE_TIMEOUT = 0, -1, -2, -3, -4, -5
 F32, BF16, FP8_E4M3_B128, INT4_G128, MXFP4 = 0, 1, 2, 3, 4
 SOFTMAX, SIGMOID = 0, 1
-FFN_AUTO, FFN_STREAM, FFN_SIMT, FFN_TC, FFN_TC_DEQUANT = 0, 1, 2, 3, 4
+FFN_AUTO, FFN_STREAM, FFN_SIMT, FFN_TC, FFN_TC_DEQUANT, FFN_TC_FP8 = 0, 1, 2, 3, 4, 5
 
 DTYPES = {"f32": F32, "bf16": BF16, "fp8_b128": FP8_E4M3_B128, "int4_g128": INT4_G128, "mxfp4": MXFP4}
-ROUTES = {"auto": FFN_AUTO, "stream": FFN_STREAM, "simt": FFN_SIMT, "tc": FFN_TC, "tc_dequant": FFN_TC_DEQUANT}
+ROUTES = {"auto": FFN_AUTO, "stream": FFN_STREAM, "simt": FFN_SIMT, "tc": FFN_TC, "tc_dequant": FFN_TC_DEQUANT,
+          "tc_fp8": FFN_TC_FP8}
 
 # every function include/gbmoe.h declares
 EXPORTS = ("gbmoe_status_string", "gbmoe_check_config", "gbmoe_workspace_size", "gbmoe_ffn_route", "moe_route",
@@ -126,7 +127,7 @@ def workspace_size(cfg: Config) -> int:
 
 
 def ffn_route(cfg: Config, shared: bool = False) -> str:
-    """Name of the FFN route moe_forward runs for cfg ("stream", "simt", "tc", "tc_dequant")."""
+    """Name of the FFN route moe_forward runs for cfg ("stream", "simt", "tc", "tc_dequant", "tc_fp8")."""
     r = lib().gbmoe_ffn_route(ctypes.byref(cfg), int(bool(shared)))
     if r < 0:
         raise GbmoeError(r, "gbmoe_ffn_route")

@@ -32,7 +32,7 @@ int check_cfg(const gbmoe_config* c) {
     if (c->w_dtype < GBMOE_F32 || c->w_dtype > GBMOE_MXFP4) return GBMOE_EINVAL;
     if (c->has_shared != 0 && c->has_shared != 1) return GBMOE_EINVAL;
     if (c->has_shared && c->I_shared <= 0) return GBMOE_EINVAL;
-    if (c->ffn_route < GBMOE_FFN_AUTO || c->ffn_route > GBMOE_FFN_TC_DEQUANT) return GBMOE_EINVAL;
+    if (c->ffn_route < GBMOE_FFN_AUTO || c->ffn_route > GBMOE_FFN_TC_FP8) return GBMOE_EINVAL;
     if (!std::isfinite(c->routed_scale)) return GBMOE_EINVAL;
     if (c->score == GBMOE_SIGMOID) {
         if (c->n_group < 1 || c->E % c->n_group != 0) return GBMOE_EINVAL;
@@ -48,6 +48,8 @@ int check_cfg(const gbmoe_config* c) {
     if ((int64_t)c->T * c->top_k > (int64_t(1) << 30)) return GBMOE_EUNSUPPORTED;
     if (c->act_dtype == GBMOE_BF16 && c->w_dtype == GBMOE_F32) return GBMOE_EUNSUPPORTED;
     if ((c->ffn_route == GBMOE_FFN_TC || c->ffn_route == GBMOE_FFN_TC_DEQUANT) && c->act_dtype != GBMOE_BF16)
+        return GBMOE_EUNSUPPORTED;
+    if (c->ffn_route == GBMOE_FFN_TC_FP8 && (c->act_dtype != GBMOE_BF16 || c->w_dtype != GBMOE_FP8_E4M3_B128))
         return GBMOE_EUNSUPPORTED;
     return GBMOE_OK;
 }
@@ -83,8 +85,14 @@ size_t dequant_bytes(const gbmoe_config* c, int64_t n_rows, int E, int I) {
 
 struct Layout {
     size_t err, logits, ids, w, counts, offsets, sorted, pos, perm, sched, h, xs, y, ysh, xin, xout, wdq, wdq_sh,
-        total;
+        aq, as, hq, hs, total;
 };
+
+// true when the routed or the shared FFN problem of c runs on the fp8 route
+bool uses_fp8_route(const gbmoe_config* c) {
+    if (pick_route(c, (int64_t)c->T * c->top_k, c->E, c->I) == GBMOE_FFN_TC_FP8) return true;
+    return c->has_shared && pick_route(c, c->T, 1, c->I_shared) == GBMOE_FFN_TC_FP8;
+}
 
 Layout layout(const gbmoe_config* c) {
     const int64_t T = c->T, P = (int64_t)c->T * c->top_k, E = c->E, H = c->H;
@@ -112,6 +120,11 @@ Layout layout(const gbmoe_config* c) {
     L.xout = take((size_t)T * H * ab);
     L.wdq = take(dequant_bytes(c, P, (int)E, c->I));
     L.wdq_sh = take(c->has_shared ? dequant_bytes(c, T, 1, c->I_shared) : 0);
+    const bool f8 = uses_fp8_route(c);  // e4m3 copies of the GEMM inputs and their 1x128 scales
+    L.aq = take(f8 ? (size_t)2 * rows_max * H : 0);  // two e4m3 code planes
+    L.as = take(f8 ? (size_t)rows_max * (H / 128) * 4 : 0);
+    L.hq = take(f8 ? (size_t)2 * rows_max * I_max : 0);
+    L.hs = take(f8 ? (size_t)rows_max * (I_max / 128) * 4 : 0);
     L.total = o;
     return L;
 }
@@ -155,13 +168,15 @@ int route_launchable(const gbmoe_config* c, int route, int I) {
         case GBMOE_FFN_STREAM: return stream_fits(c->act_dtype, c->H, I) ? GBMOE_OK : GBMOE_EUNSUPPORTED;
         case GBMOE_FFN_SIMT: return GBMOE_OK;
         case GBMOE_FFN_TC:
-        case GBMOE_FFN_TC_DEQUANT: {
+        case GBMOE_FFN_TC_DEQUANT:
+        case GBMOE_FFN_TC_FP8: {
             FfnProblem probe{};
             probe.act_dtype = c->act_dtype;
             probe.w_dtype = c->w_dtype;
             probe.H = c->H;
             probe.I = I;
-            return ffn_tc_supported(probe) ? GBMOE_OK : GBMOE_EUNSUPPORTED;
+            const bool ok = route == GBMOE_FFN_TC_FP8 ? ffn_tc_fp8_supported(probe) : ffn_tc_supported(probe);
+            return ok ? GBMOE_OK : GBMOE_EUNSUPPORTED;
         }
         default: return GBMOE_EINVAL;
     }
@@ -173,9 +188,19 @@ int run_ffn(const gbmoe_config* c, FfnProblem& p, int route, cudaStream_t stream
     switch (route) {
         case GBMOE_FFN_STREAM: err = launch_ffn_stream(p, stream); break;
         case GBMOE_FFN_SIMT: err = launch_ffn_simt(p, stream); break;
+        case GBMOE_FFN_TC_FP8: err = launch_ffn_tc_fp8(p, stream); break;
         default: err = launch_ffn_tc(p, stream); break;  // GBMOE_FFN_TC, GBMOE_FFN_TC_DEQUANT
     }
     return cuda_status(err);
+}
+
+// the fp8 route's scratch (the routed and the shared problem run one after
+// the other, so they share it)
+void set_fp8_buffers(FfnProblem& p, const Layout& L, void* ws) {
+    p.a_q = at<char>(ws, L.aq);
+    p.a_s = at<float>(ws, L.as);
+    p.h_q = at<char>(ws, L.hq);
+    p.h_s = at<float>(ws, L.hs);
 }
 
 FfnProblem routed_problem(const gbmoe_config* c, const void* x, const int32_t* counts, const int32_t* offsets,
@@ -191,6 +216,7 @@ FfnProblem routed_problem(const gbmoe_config* c, const void* x, const int32_t* c
     p.h = at<char>(ws, L.h); p.x_sorted = at<char>(ws, L.xs); p.sched = at<int32_t>(ws, L.sched);
     p.err = at<int32_t>(ws, L.err);
     p.w_dq = dequant_bytes(c, p.n_rows, p.E, p.I) ? at<char>(ws, L.wdq) : nullptr;
+    set_fp8_buffers(p, L, ws);
     return p;
 }
 
@@ -206,6 +232,7 @@ FfnProblem shared_problem(const gbmoe_config* c, const void* x, const gbmoe_expe
     p.h = at<char>(ws, L.h); p.x_sorted = at<char>(ws, L.xs); p.sched = at<int32_t>(ws, L.sched);
     p.err = at<int32_t>(ws, L.err);
     p.w_dq = dequant_bytes(c, p.n_rows, p.E, p.I) ? at<char>(ws, L.wdq_sh) : nullptr;
+    set_fp8_buffers(p, L, ws);
     return p;
 }
 

@@ -43,6 +43,11 @@ struct FfnProblem {
     void* x_sorted;             // [n_rows, H] act (tensor-core route only)
     void* w_dq;                 // bf16 [E, I, H] gate, [E, I, H] up, [E, H, I] down, or null:
                                 // quantised weights are then decoded once into it (TC_DEQUANT)
+    void* a_q;                  // fp8 route (TC_FP8): x rows in sorted order as two e4m3 code planes
+                                //   [2, n_rows, H] (value and residual)
+    float* a_s;                 //   and their 1x128 scales [n_rows, H/128]
+    void* h_q;                  //   h the same way, [2, n_rows, I]
+    float* h_s;                 //   and its 1x128 scales [n_rows, I/128]
     int32_t* sched;             // schedule ints, ffn_sched_ints(E, n_rows)
     int32_t* err;               // device error word
 };
@@ -57,6 +62,8 @@ constexpr size_t stream_smem_budget() { return 227 * 1024; }
 cudaError_t launch_ffn_simt(const FfnProblem& p, cudaStream_t stream);
 cudaError_t launch_ffn_tc(const FfnProblem& p, cudaStream_t stream);
 bool ffn_tc_supported(const FfnProblem& p);
+cudaError_t launch_ffn_tc_fp8(const FfnProblem& p, cudaStream_t stream);
+bool ffn_tc_fp8_supported(const FfnProblem& p);
 
 cudaError_t launch_combine(const void* y_pairs, const float* topk_w, const int32_t* pair_pos, const void* y_shared,
                            void* out, int T, int k, int H, int act_dtype, cudaStream_t stream);

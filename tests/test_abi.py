@@ -70,6 +70,8 @@ def test_workload_configs_are_valid(lib, wid):
     (dict(ffn_route=9), gb.EINVAL),
     (dict(ffn_route=gb.FFN_TC), gb.EUNSUPPORTED),  # fp32 activations have no tensor-core route
     (dict(ffn_route=gb.FFN_TC_DEQUANT), gb.EUNSUPPORTED),
+    (dict(ffn_route=gb.FFN_TC_FP8), gb.EUNSUPPORTED),  # fp8 route needs fp8 weights and bf16 activations
+    (dict(ffn_route=6), gb.EINVAL),
 ])
 def test_invalid_configs_are_rejected(lib, change, status):
     c = cfg_of(1, **change)
@@ -83,6 +85,8 @@ def test_sigmoid_group_rules(lib):
         bad = cfg_of(4, **ch)
         assert gb.check_config(bad) == gb.EINVAL, ch
     assert gb.check_config(c) == gb.OK
+    assert gb.check_config(cfg_of(4, ffn_route=gb.FFN_TC_FP8)) == gb.OK
+    assert gb.check_config(cfg_of(5, ffn_route=gb.FFN_TC_FP8)) == gb.EUNSUPPORTED  # int4 weights
 
 
 class FakePtr:

@@ -2,6 +2,8 @@
 oracle on small ragged problems (the full-size workloads are compared token
 by token in test_gpu_layer.py), and the decode-once route (TC_DEQUANT)
 against the in-GEMM decode."""
+import os
+
 import numpy as np
 import pytest
 import torch
@@ -118,3 +120,43 @@ def test_bounded_wait_timeout_is_reported_and_the_next_call_is_clean(wq, monkeyp
     assert gb.moe_device_status(ws) == gb.OK
     ref = oracle.forward(wl, inp)
     assert_close(act_np(out), ref["out"], tol_for(wl))
+
+
+# fp8 tensor-core route (kind::f8f6f4): fp8 weights as stored, activations
+# quantised to e4m3 per 1x128 block; against the oracle with exact
+# activations, within the fp8 bound (5e-2) and per row
+@pytest.mark.parametrize("T,E,k,H,I", [(200, 4, 2, 512, 256), (1000, 4, 2, 256, 384), (333, 16, 3, 768, 128),
+                                       (64, 8, 8, 1024, 512)])
+def test_tc_fp8_route_small_ragged(T, E, k, H, I):
+    wl = BASE.replace(T=T, E=E, top_k=k, H=H, I=I, seed=T + 3 * E, wq="fp8_b128")
+    inp = synth.make_inputs(wl)
+    dev = to_device(wl, inp)
+    out, ids = forward(wl, dev, "tc_fp8")
+    ref = oracle.forward(wl, inp)
+    assert np.array_equal(ids.cpu().numpy(), ref["topk_ids"])
+    assert_close(act_np(out), ref["out"], tol_for(wl))
+
+
+def test_tc_fp8_route_with_shared_expert_and_timeout():
+    """Sigmoid group routing with a shared expert on the fp8 route; then its
+    bounded waits run out under a 0 ns limit and the next call is clean."""
+    wl = BASE.replace(T=300, E=16, top_k=4, H=512, I=256, wq="fp8_b128", seed=33, score="sigmoid",
+                      routed_scale=2.5, n_group=4, topk_group=2, has_shared=True, I_shared=384,
+                      select_bias_sigma=0.01)
+    inp = synth.make_inputs(wl)
+    dev = to_device(wl, inp)
+    out, ids = forward(wl, dev, "tc_fp8")
+    ref = oracle.forward(wl, inp)
+    assert np.array_equal(ids.cpu().numpy(), ref["topk_ids"])
+    assert_close(act_np(out), ref["out"], tol_for(wl))
+    cfg = config(wl, "tc_fp8")
+    ws = workspace(cfg)
+    os.environ["GBMOE_TC_WAIT_LIMIT_NS"] = "0"
+    try:
+        gb.moe_forward(cfg, dev["x"], dev["w_router"], dev["logit_bias"], dev["select_bias"],
+                       wbundle(dev["experts"]), wbundle(dev["shared"]), out, ws)
+        assert gb.moe_device_status(ws) == gb.EDEVICE_TIMEOUT
+    finally:
+        del os.environ["GBMOE_TC_WAIT_LIMIT_NS"]
+    out2, _ = forward(wl, dev, "tc_fp8")
+    assert_close(act_np(out2), ref["out"], tol_for(wl))
