@@ -252,6 +252,8 @@ def launches_per_step(wl, route: str, shared_route) -> int:
     routed experts on the tensor-core routes, + 3 weight-decode passes on the
     decode-once route), and the combine."""
     def ffn(r, routed):
+        if r == "tc_fp8":  # schedule, x quantisation, gate/up GEMM, h quantisation, down GEMM
+            return 5
         return 3 + (1 if routed and r in ("tc", "tc_dequant") else 0) + (3 if r == "tc_dequant" else 0)
 
     n = 2 + (1 if wl.P <= 1024 else 3) + ffn(route, True) + 1

@@ -64,17 +64,18 @@ enum {
 enum { GBMOE_SOFTMAX = 0, GBMOE_SIGMOID = 1 };
 
 /* Which expert-FFN kernels run. GBMOE_FFN_TC_FP8 (FP8_E4M3_B128 weights and
- * bf16 activations only) follows the DeepSeek-V3 recipe: each GEMM's input
- * rows (x, then h) are quantised to e4m3 with one fp32 scale per row and 128
- * consecutive k (scale = amax / 448, round to nearest even), the tensor cores
- * multiply e4m3 by e4m3, and each 128-wide k block's partial sum is scaled by
- * both blocks' scales and accumulated in fp32. The activation rounding makes
- * its outputs differ from the other routes' by about 1-3% of their typical
- * magnitude (the fp8 tolerance, 5e-2 of the largest output, covers it).
+ * bf16 activations only) multiplies the stored e4m3 weights on the fp8 tensor
+ * cores: each GEMM's input rows (x, then h) are brought to e4m3 with one fp32
+ * scale s per row and 128 consecutive k (s = amax / 448) as two codes,
+ * q1 = e4m3(x / s) and q2 = e4m3(x / s - q1), so that x = s * (q1 + q2) to
+ * within max(2^-8 |x / s|, 2^-10) * s, a bf16-like precision; both codes are
+ * multiplied with the weights and each 128-wide k block's partial sum is
+ * scaled by both blocks' scales and accumulated in fp32. AUTO takes it for
+ * fp8 weights whenever a tensor-core route applies.
  * AUTO streams weights when the average number
  * of rows per expert P/E is at most 16 and otherwise runs the grouped GEMM
  * (tensor cores for bf16 activations, CUDA cores for fp32). On the tensor
- * cores, fp8/int4/MXFP4 weights are decoded inside the GEMM when P/E < 256; with
+ * cores, int4/MXFP4 weights are decoded inside the GEMM when P/E < 256; with
  * more rows per expert (several M tiles reuse each weight tile) AUTO takes
  * GBMOE_FFN_TC_DEQUANT: one pass decodes the active experts' weights to a
  * bf16 copy in the workspace (the same bf16 values the in-GEMM decode makes),

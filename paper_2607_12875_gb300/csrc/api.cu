@@ -68,6 +68,9 @@ int pick_route(const gbmoe_config* c, int64_t n_rows, int E, int I) {
         probe.H = c->H;
         probe.I = I;
         probe.E = E;
+        // fp8 weights: the fp8 tensor-core route (no decode; its two-term
+        // activation codes keep bf16-level accuracy)
+        if (ffn_tc_fp8_supported(probe)) return GBMOE_FFN_TC_FP8;
         if (ffn_tc_supported(probe)) {
             return quantised_weights(c->w_dtype) && n_rows >= kDequantRowsPerExpert * E ? GBMOE_FFN_TC_DEQUANT
                                                                                         : GBMOE_FFN_TC;

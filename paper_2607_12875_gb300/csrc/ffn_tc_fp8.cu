@@ -151,30 +151,39 @@ quant_rows_kernel(const __nv_bfloat16* __restrict__ src, const int32_t* __restri
             const int32_t pr = sorted_pair[r];
             srow = pr >= 0 ? pr / pair_div : -1;
         }
-        for (int b = 0; b < nblk; ++b) {
-            float v[4] = {0.f, 0.f, 0.f, 0.f};
-            if (srow >= 0) {
-                const uint2 u = *reinterpret_cast<const uint2*>(src + srow * K + b * QB + 4 * lane);
-                v[0] = bf16lo(u.x); v[1] = bf16hi(u.x); v[2] = bf16lo(u.y); v[3] = bf16hi(u.y);
+        constexpr int U = 8;  // blocks whose loads are in flight together
+        for (int b0 = 0; b0 < nblk; b0 += U) {
+            uint2 raw[U];
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                raw[u] = make_uint2(0, 0);
+                if (srow >= 0 && b0 + u < nblk)
+                    raw[u] = *reinterpret_cast<const uint2*>(src + srow * K + (b0 + u) * QB + 4 * lane);
             }
-            float amax = fmaxf(fmaxf(fabsf(v[0]), fabsf(v[1])), fmaxf(fabsf(v[2]), fabsf(v[3])));
 #pragma unroll
-            for (int d = 16; d >= 1; d >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, d));
-            const float sc = amax > 0.0f ? __fdiv_rn(amax, 448.0f) : 1.0f;
-            float t[4], rr[4];
+            for (int u = 0; u < U; ++u) {
+                const int b = b0 + u;
+                if (b >= nblk) break;
+                const float v[4] = {bf16lo(raw[u].x), bf16hi(raw[u].x), bf16lo(raw[u].y), bf16hi(raw[u].y)};
+                float amax = fmaxf(fmaxf(fabsf(v[0]), fabsf(v[1])), fmaxf(fabsf(v[2]), fabsf(v[3])));
 #pragma unroll
-            for (int i = 0; i < 4; ++i) t[i] = __fdiv_rn(v[i], sc);
-            const uint32_t a01 = e4m3x2(t[0], t[1]), a23 = e4m3x2(t[2], t[3]);
-            const uint32_t a = a01 | (a23 << 16);
+                for (int d = 16; d >= 1; d >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, d));
+                const float sc = amax > 0.0f ? __fdiv_rn(amax, 448.0f) : 1.0f;
+                float t[4], rr[4];
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const __half_raw h = __nv_cvt_fp8_to_halfraw((__nv_fp8_storage_t)((a >> (8 * i)) & 0xffu), __NV_E4M3);
-                rr[i] = __fsub_rn(t[i], __half2float(__half(h)));
+                for (int i = 0; i < 4; ++i) t[i] = __fdiv_rn(v[i], sc);
+                const uint32_t a = e4m3x2(t[0], t[1]) | (e4m3x2(t[2], t[3]) << 16);
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const __half_raw h =
+                        __nv_cvt_fp8_to_halfraw((__nv_fp8_storage_t)((a >> (8 * i)) & 0xffu), __NV_E4M3);
+                    rr[i] = __fsub_rn(t[i], __half2float(__half(h)));
+                }
+                const uint32_t a2 = e4m3x2(rr[0], rr[1]) | (e4m3x2(rr[2], rr[3]) << 16);
+                *reinterpret_cast<uint32_t*>(q1 + r * K + b * QB + 4 * lane) = a;
+                *reinterpret_cast<uint32_t*>(q2 + r * K + b * QB + 4 * lane) = a2;
+                if (lane == 0) s[r * nblk + b] = sc;
             }
-            const uint32_t a2 = e4m3x2(rr[0], rr[1]) | (e4m3x2(rr[2], rr[3]) << 16);
-            *reinterpret_cast<uint32_t*>(q1 + r * K + b * QB + 4 * lane) = a;
-            *reinterpret_cast<uint32_t*>(q2 + r * K + b * QB + 4 * lane) = a2;
-            if (lane == 0) s[r * nblk + b] = sc;
         }
     }
 }
@@ -316,11 +325,23 @@ tc_fp8_gemm_kernel(const __grid_constant__ CUtensorMap tm_a1, const __grid_const
             float acc[128];
 #pragma unroll
             for (int i = 0; i < 128; ++i) acc[i] = 0.0f;
+            // the k block's scales, loaded two k blocks ahead so that the
+            // promotion never waits on a global load
+            auto scales_of = [&](int kb, float& a, float& w0, float& w1) {
+                const bool ok_kb = kb < nkb;
+                a = in_range && ok_kb ? sa[kb] : 0.0f;
+                w0 = ok_kb ? s0[kb] : 0.0f;
+                w1 = ok_kb ? s1[kb] : 0.0f;
+            };
+            float a0, x0, y0, a1, x1, y1;
+            scales_of(0, a0, x0, y0);
+            scales_of(1, a1, x1, y1);
             bool ok = true;
             for (int kb = 0; kb < nkb; ++kb, ++kbg) {
                 const uint32_t pb = kbg & 1u, pph = (kbg >> 1) & 1u;
-                const float a_s = in_range ? sa[kb] : 0.0f;
-                const float f0 = a_s * s0[kb], f1 = a_s * s1[kb];
+                const float f0 = a0 * x0, f1 = a0 * y0;
+                a0 = a1; x0 = x1; y0 = y1;
+                scales_of(kb + 2, a1, x1, y1);
                 if (!warp_wait(&pfull[pb], pph, abort_flag, p.err, p.wait_limit_ns)) { ok = false; break; }
                 tc_fence_after();
                 const uint32_t tb = t_row + pb * BN;

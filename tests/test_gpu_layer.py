@@ -19,7 +19,7 @@ from gpu_helpers import (act_np, assert_close, config, rel_err, tiles_covered, t
 pytestmark = pytest.mark.gpu
 
 ROUTES = {1: ["simt", "stream", "auto"], 2: ["stream", "simt", "auto"], 3: ["simt", "auto"],
-          4: ["simt", "auto", "tc_dequant", "tc_fp8"], 5: ["simt", "auto", "tc"], 6: ["simt", "auto", "tc_dequant"]}
+          4: ["simt", "auto", "tc", "tc_dequant"], 5: ["simt", "auto", "tc"], 6: ["simt", "auto", "tc_dequant"]}
 ALL_ROUTES = ["auto", "stream", "simt", "tc", "tc_dequant", "tc_fp8"]
 
 

@@ -84,12 +84,13 @@ def test_dequant_route_with_shared_expert_and_inactive_experts():
 
 
 def test_auto_route_choice():
-    """AUTO: streaming for decode, in-GEMM decode for few rows per expert,
-    decode-once for many."""
+    """AUTO: streaming for decode; fp8 weights on the fp8 tensor-core route;
+    int4/MXFP4 decoded in the GEMM for few rows per expert, decoded once for
+    many."""
     assert gb.ffn_route(config(synth.WORKLOADS[2])) == "stream"
     assert gb.ffn_route(config(synth.WORKLOADS[3])) == "tc"
-    assert gb.ffn_route(config(synth.WORKLOADS[4])) == "tc"
-    assert gb.ffn_route(config(synth.WORKLOADS[4]), shared=True) == "tc_dequant"
+    assert gb.ffn_route(config(synth.WORKLOADS[4])) == "tc_fp8"
+    assert gb.ffn_route(config(synth.WORKLOADS[4]), shared=True) == "tc_fp8"
     assert gb.ffn_route(config(synth.WORKLOADS[5])) == "tc_dequant"
     assert gb.ffn_route(config(synth.WORKLOADS[6])) == "tc"
     assert gb.ffn_route(config(synth.WORKLOADS[6]), shared=True) == "tc_dequant"
