@@ -90,6 +90,22 @@ enum {
                                  activations quantised to e4m3 per 1x128 block      */
 };
 
+/* How the MoE Gate computes the router logits. SIMT: CUDA cores in the fixed
+ * order of the definition (moe_route). TC: tensor cores (bf16 activations
+ * only), whose fp32 sums run in the hardware's order; each token's expert
+ * choice is then audited: when any comparison that decides it (the order of
+ * the chosen keys, the chosen against the best one left out, and the last
+ * kept group against the best dropped one) is closer than a bound on the
+ * difference between the two orders (scale * ||x_t|| * max_e ||w_e||, plus a
+ * few units in the last place), that token's logits are recomputed in the
+ * fixed order and its choice is made again, so the ids equal the SIMT
+ * route's. The scale (2e-6) is four times the largest difference measured on
+ * the benchmark workloads, not a worst-case bound. The routing weights of
+ * tokens not recomputed come from the tensor-core logits: within about 1e-4
+ * relative of the SIMT route's. AUTO: TC for bf16 batches of 256 tokens or
+ * more, else SIMT. */
+enum { GBMOE_GATE_AUTO = 0, GBMOE_GATE_SIMT = 1, GBMOE_GATE_TC = 2 };
+
 typedef struct gbmoe_config {
     int32_t T, H, I, E, top_k;
     int32_t score;        /* GBMOE_SOFTMAX or GBMOE_SIGMOID                         */
@@ -102,6 +118,7 @@ typedef struct gbmoe_config {
     int32_t has_shared;   /* 1: add one always-on expert with weight 1              */
     int32_t I_shared;     /* its intermediate size                                  */
     int32_t ffn_route;    /* GBMOE_FFN_*                                            */
+    int32_t gate_route;   /* GBMOE_GATE_*                                           */
 } gbmoe_config;
 
 /* One set of expert weights (all experts stacked, E of them, or 1 for the
@@ -144,6 +161,10 @@ size_t gbmoe_workspace_size(const gbmoe_config* cfg);
  * cfg: for the routed experts (shared = 0) or the shared expert (shared = 1).
  * Negative status if the config is invalid. */
 int gbmoe_ffn_route(const gbmoe_config* cfg, int shared);
+
+/* The gate route (GBMOE_GATE_SIMT or _TC) that moe_route and moe_forward run
+ * for cfg. Negative status if the config is invalid. */
+int gbmoe_gate_route(const gbmoe_config* cfg);
 
 /*
  * MoE Gate (Fig. 1 and Fig. 3). For every token t:

@@ -20,13 +20,16 @@ OK, EINVAL, EUNSUPPORTED, EWORKSPACE, ECUDA, EDEVICE_TIMEOUT = 0, -1, -2, -3, -4
 F32, BF16, FP8_E4M3_B128, INT4_G128, MXFP4 = 0, 1, 2, 3, 4
 SOFTMAX, SIGMOID = 0, 1
 FFN_AUTO, FFN_STREAM, FFN_SIMT, FFN_TC, FFN_TC_DEQUANT, FFN_TC_FP8 = 0, 1, 2, 3, 4, 5
+GATE_AUTO, GATE_SIMT, GATE_TC = 0, 1, 2
 
 DTYPES = {"f32": F32, "bf16": BF16, "fp8_b128": FP8_E4M3_B128, "int4_g128": INT4_G128, "mxfp4": MXFP4}
+GATES = {"auto": GATE_AUTO, "simt": GATE_SIMT, "tc": GATE_TC}
 ROUTES = {"auto": FFN_AUTO, "stream": FFN_STREAM, "simt": FFN_SIMT, "tc": FFN_TC, "tc_dequant": FFN_TC_DEQUANT,
           "tc_fp8": FFN_TC_FP8}
 
 # every function include/gbmoe.h declares
-EXPORTS = ("gbmoe_status_string", "gbmoe_check_config", "gbmoe_workspace_size", "gbmoe_ffn_route", "moe_route",
+EXPORTS = ("gbmoe_status_string", "gbmoe_check_config", "gbmoe_workspace_size", "gbmoe_ffn_route",
+           "gbmoe_gate_route", "moe_route",
            "moe_permute",
            "moe_grouped_ffn", "moe_shared_ffn", "moe_combine", "moe_forward", "moe_forward_hostio",
            "moe_device_status", "moe_permute_noalloc")
@@ -43,7 +46,7 @@ class Config(ctypes.Structure):
                 ("top_k", ctypes.c_int32), ("score", ctypes.c_int32), ("renormalize", ctypes.c_int32),
                 ("n_group", ctypes.c_int32), ("topk_group", ctypes.c_int32), ("routed_scale", ctypes.c_float),
                 ("act_dtype", ctypes.c_int32), ("w_dtype", ctypes.c_int32), ("has_shared", ctypes.c_int32),
-                ("I_shared", ctypes.c_int32), ("ffn_route", ctypes.c_int32)]
+                ("I_shared", ctypes.c_int32), ("ffn_route", ctypes.c_int32), ("gate_route", ctypes.c_int32)]
 
 
 class ExpertWeights(ctypes.Structure):
@@ -70,6 +73,7 @@ def lib() -> ctypes.CDLL:
         L.gbmoe_workspace_size.argtypes = [cfgp]
         L.gbmoe_workspace_size.restype = sz
         L.gbmoe_ffn_route.argtypes = [cfgp, ctypes.c_int]
+        L.gbmoe_gate_route.argtypes = [cfgp]
         L.moe_route.argtypes = [cfgp, vp, vp, fp, fp, vp, vp, vp, sz, vp]
         L.moe_permute.argtypes = [cfgp, vp, vp, vp, vp, vp, vp, sz, vp]
         L.moe_grouped_ffn.argtypes = [cfgp, vp, vp, vp, vp, wp, vp, vp, sz, vp]
@@ -88,10 +92,11 @@ def status_string(status: int) -> str:
 
 
 def make_config(T, H, I, E, top_k, *, score="softmax", renormalize=True, n_group=1, topk_group=1,
-                routed_scale=1.0, act="bf16", w="bf16", has_shared=False, I_shared=0, ffn_route="auto") -> Config:
+                routed_scale=1.0, act="bf16", w="bf16", has_shared=False, I_shared=0, ffn_route="auto",
+                gate_route="auto") -> Config:
     return Config(T, H, I, E, top_k, SOFTMAX if score == "softmax" else SIGMOID, int(bool(renormalize)), n_group,
                   topk_group, routed_scale, DTYPES[act], DTYPES[w], int(bool(has_shared)), I_shared,
-                  ROUTES[ffn_route])
+                  ROUTES[ffn_route], GATES[gate_route])
 
 
 def _ptr(t):
@@ -116,6 +121,14 @@ def _check(status: int, call: str) -> None:
 def weights(w_gate, w_up, w_down, s_gate=None, s_up=None, s_down=None) -> ExpertWeights:
     """Pointer bundle of one set of expert weights (tensors must stay alive)."""
     return ExpertWeights(_ptr(w_gate), _ptr(w_up), _ptr(w_down), _ptr(s_gate), _ptr(s_up), _ptr(s_down))
+
+
+def gate_route(cfg: Config) -> str:
+    """Name of the gate route moe_route runs for cfg ("simt" or "tc")."""
+    r = lib().gbmoe_gate_route(ctypes.byref(cfg))
+    if r < 0:
+        raise GbmoeError(r, "gbmoe_gate_route")
+    return {v: k for k, v in GATES.items()}[r]
 
 
 def check_config(cfg: Config) -> int:

@@ -33,6 +33,8 @@ int check_cfg(const gbmoe_config* c) {
     if (c->has_shared != 0 && c->has_shared != 1) return GBMOE_EINVAL;
     if (c->has_shared && c->I_shared <= 0) return GBMOE_EINVAL;
     if (c->ffn_route < GBMOE_FFN_AUTO || c->ffn_route > GBMOE_FFN_TC_FP8) return GBMOE_EINVAL;
+    if (c->gate_route < GBMOE_GATE_AUTO || c->gate_route > GBMOE_GATE_TC) return GBMOE_EINVAL;
+    if (c->gate_route == GBMOE_GATE_TC && c->act_dtype != GBMOE_BF16) return GBMOE_EUNSUPPORTED;
     if (!std::isfinite(c->routed_scale)) return GBMOE_EINVAL;
     if (c->score == GBMOE_SIGMOID) {
         if (c->n_group < 1 || c->E % c->n_group != 0) return GBMOE_EINVAL;
@@ -87,8 +89,8 @@ size_t dequant_bytes(const gbmoe_config* c, int64_t n_rows, int E, int I) {
 }
 
 struct Layout {
-    size_t err, logits, ids, w, counts, offsets, sorted, pos, perm, sched, h, xs, y, ysh, xin, xout, wdq, wdq_sh,
-        aq, as, hq, hs, total;
+    size_t err, audit, flagged, logits, ids, w, counts, offsets, sorted, pos, perm, sched, h, xs, y, ysh, xin, xout, wdq,
+        wdq_sh, aq, as, hq, hs, total;
 };
 
 // true when the routed or the shared FFN problem of c runs on the fp8 route
@@ -106,6 +108,8 @@ Layout layout(const gbmoe_config* c) {
     size_t o = 0;
     auto take = [&](size_t bytes) { size_t at = o; o = align_up(o + bytes); return at; };
     L.err = take(4);
+    L.audit = take(8);
+    L.flagged = take((size_t)T * 4);
     L.logits = take((size_t)T * E * 4);
     L.ids = take((size_t)P * 4);
     L.w = take((size_t)P * 4);
@@ -156,12 +160,34 @@ int check_weights(const gbmoe_config* c, const gbmoe_expert_weights* w) {
     return GBMOE_OK;
 }
 
+// Gate route: the fixed-order CUDA-core logits, or tensor-core logits audited
+// against that order (AUTO: bf16 batches of at least kGateTcMinTokens tokens).
+constexpr int kGateTcMinTokens = 256;
+
+int pick_gate(const gbmoe_config* c) {
+    if (c->gate_route != GBMOE_GATE_AUTO) return c->gate_route;
+    if (c->act_dtype != GBMOE_BF16 || c->T < kGateTcMinTokens) return GBMOE_GATE_SIMT;
+    FfnProblem probe{};
+    probe.act_dtype = c->act_dtype;
+    probe.w_dtype = GBMOE_BF16;
+    probe.H = c->H;
+    probe.I = 128;
+    return ffn_tc_supported(probe) ? GBMOE_GATE_TC : GBMOE_GATE_SIMT;
+}
+
 RouteParams route_params(const gbmoe_config* c) {
     RouteParams rp;
     rp.T = c->T; rp.H = c->H; rp.E = c->E; rp.top_k = c->top_k;
     rp.score = c->score; rp.renormalize = c->renormalize; rp.n_group = c->n_group;
     rp.topk_group = c->topk_group; rp.routed_scale = c->routed_scale; rp.act_dtype = c->act_dtype;
+    rp.gate_tc = pick_gate(c) == GBMOE_GATE_TC;
     return rp;
+}
+
+RouteScratch route_scratch(const gbmoe_config* c, void* ws) {
+    const Layout L = layout(c);
+    return RouteScratch{at<int32_t>(ws, L.sched), at<int32_t>(ws, L.err), at<float>(ws, L.audit),
+                        at<int32_t>(ws, L.flagged)};
 }
 
 // GBMOE_OK when an FFN problem of intermediate size I can run on `route`,
@@ -269,6 +295,11 @@ int gbmoe_ffn_route(const gbmoe_config* cfg, int shared) {
     return pick_route(cfg, (int64_t)cfg->T * cfg->top_k, cfg->E, cfg->I);
 }
 
+int gbmoe_gate_route(const gbmoe_config* cfg) {
+    int s = check_cfg(cfg);
+    return s ? s : pick_gate(cfg);
+}
+
 int moe_route(const gbmoe_config* cfg, const void* x, const void* w_router, const float* logit_bias,
               const float* select_bias, int32_t* topk_ids, float* topk_w, void* ws, size_t ws_bytes,
               void* stream) {
@@ -282,7 +313,7 @@ int moe_route(const gbmoe_config* cfg, const void* x, const void* w_router, cons
     if ((s = check_ws(cfg, ws, ws_bytes))) return s;
     const Layout L = layout(cfg);
     return cuda_status(launch_route(route_params(cfg), x, w_router, logit_bias, select_bias, at<float>(ws, L.logits),
-                                    topk_ids, topk_w, static_cast<cudaStream_t>(stream)));
+                                    topk_ids, topk_w, route_scratch(cfg, ws), static_cast<cudaStream_t>(stream)));
 }
 
 int moe_permute(const gbmoe_config* cfg, const int32_t* topk_ids, int32_t* counts, int32_t* offsets,
@@ -373,7 +404,7 @@ int moe_forward(const gbmoe_config* cfg, const void* x, const void* w_router, co
     int32_t* sorted = at<int32_t>(ws, L.sorted);
     int32_t* pos = at<int32_t>(ws, L.pos);
     if ((s = cuda_status(launch_route(route_params(cfg), x, w_router, logit_bias, select_bias,
-                                      at<float>(ws, L.logits), ids, w, st))))
+                                      at<float>(ws, L.logits), ids, w, route_scratch(cfg, ws), st))))
         return s;
     if ((s = cuda_status(launch_permute(ids, P, cfg->E, counts, offsets, sorted, pos, at<int32_t>(ws, L.perm), st))))
         return s;

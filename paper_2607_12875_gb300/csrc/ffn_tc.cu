@@ -107,6 +107,11 @@ struct Params {
     const void* scale0;  // scales of the B rows in the first / second half of the tile
     const void* scale1;
     uint64_t wait_limit_ns;  // limit of each pipeline wait (kWaitLimitNs unless a test shortens it)
+    // fp32 output instead of bf16 (the router's logits): out_f32[row, col] =
+    // accumulator (+ col_bias[col]) for col < f32_cols; out is unused then
+    float* out_f32;
+    const float* col_bias;
+    int f32_cols;
 };
 
 // Instruction descriptor, kind::f16: fp32 accumulator (bits 4-5 = 1), bf16 A
@@ -395,7 +400,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
             // all 32 rows of this warp belong to the tile: one TMA store per 32 columns;
             // otherwise plain stores of the valid rows only (the rows past the tile's end
             // belong to the next expert and are written by another tile)
-            const bool via_tma = L::EPI_BYTES > 0 && q * 32 + 32 <= wk.rows;
+            const bool via_tma = L::EPI_BYTES > 0 && q * 32 + 32 <= wk.rows && p.out_f32 == nullptr;
             const int col0 = p.swiglu ? wk.nt * (BN / 2) : wk.nt * BN;
             __nv_bfloat16* dst = p.out + (wk.row0 + r) * (int64_t)p.out_cols + col0;
             const int ncols = p.swiglu ? BN / 2 : BN;
@@ -418,6 +423,13 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
                     __syncwarp();
                     if (lane == 0) tma_store_2d(&tm_out, buf, col0 + c, (int)(wk.row0 + q * 32));
                     sbuf ^= 1;
+                } else if (valid && p.out_f32) {
+                    float* dst32 = p.out_f32 + (wk.row0 + r) * (int64_t)p.out_cols + col0 + c;
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) {
+                        const int col = col0 + c + i;
+                        if (col < p.f32_cols) dst32[i] = p.col_bias ? __fadd_rn(v[i], p.col_bias[col]) : v[i];
+                    }
                 } else if (valid) {
                     store_bf16x32(dst + c, v);
                 }
@@ -674,6 +686,28 @@ static cudaError_t dequant_all(const FfnProblem& p, FfnProblem& q, cudaStream_t 
     q.s_gate = q.s_up = q.s_down = nullptr;
     q.w_dq = nullptr;
     return cudaSuccess;
+}
+
+// Router logits on the tensor cores: logits[t, e] = x[t, :] . wg[e, :]
+// (+ bias[e]), x [T, H] and wg [E, H] bf16, fp32 accumulation in the tensor
+// core's own order (the caller audits near ties against the fixed order).
+// sched: schedule ints for one problem of T rows.
+cudaError_t launch_gate_tc(const void* x, const void* wg, const float* bias, float* logits, int T, int H, int E,
+                           int32_t* sched, int32_t* err, cudaStream_t stream) {
+    using namespace tc;
+    if (T == 0) return cudaSuccess;
+    cudaError_t e = launch_ffn_schedule(nullptr, 1, T, BM, sched, stream);
+    if (e != cudaSuccess) return e;
+    CUtensorMap ma, mb, mo;
+    // (mo is a placeholder: the fp32 epilogue stores from registers)
+    if (!map_bf16(&ma, x, T, H) || !map_bf16(&mb, wg, E, H) || !map_out(&mo, x, T, H)) return cudaErrorInvalidValue;
+    Params g{};
+    g.K = H; g.n_tiles = (E + BN - 1) / BN; g.out_cols = E; g.b_rows_per_expert = 0; g.swiglu = 0;
+    g.counts = nullptr; g.offsets = nullptr; g.sched = sched; g.E = 1; g.n_rows = T;
+    g.out = nullptr; g.err = err; g.scale0 = g.scale1 = nullptr;
+    g.wait_limit_ns = tc_wait_limit_ns();
+    g.out_f32 = logits; g.col_bias = bias; g.f32_cols = E;
+    return launch_gemm(GBMOE_BF16, ma, mb, mb, mo, g, sched_max_tiles(1, T, BM) * g.n_tiles, stream);
 }
 
 cudaError_t launch_ffn_tc(const FfnProblem& pin, cudaStream_t stream) {

@@ -11,12 +11,26 @@ struct RouteParams {
     int score, renormalize, n_group, topk_group;
     float routed_scale;
     int act_dtype;
+    int gate_tc;  // 1: logits on the tensor cores, audited against the fixed order
+};
+
+// scratch of the tensor-core gate: schedule ints for T rows, the device error
+// word, two words for the audit (max router row norm, count of flagged
+// tokens) and the list of flagged tokens [T]
+struct RouteScratch {
+    int32_t* sched;
+    int32_t* err;
+    float* audit;
+    int32_t* flagged;
 };
 
 // logits [T, E] fp32 scratch; topk_ids, topk_w [T, k]
 cudaError_t launch_route(const RouteParams& rp, const void* x, const void* w_router, const float* logit_bias,
                          const float* select_bias, float* logits, int32_t* topk_ids, float* topk_w,
-                         cudaStream_t stream);
+                         const RouteScratch& rs, cudaStream_t stream);
+// router logits on the tensor cores (bf16 x and router weight; ffn_tc.cu)
+cudaError_t launch_gate_tc(const void* x, const void* wg, const float* bias, float* logits, int T, int H, int E,
+                           int32_t* sched, int32_t* err, cudaStream_t stream);
 
 // Number of 1024-pair blocks the permutation uses, and its scratch ints.
 int permute_blocks(int64_t P);

@@ -8,6 +8,8 @@
 // of chunks l, l+32, ... for all of them, which is exactly the fixed order.
 // select_experts then runs one warp per token over the logits. Large batches
 // use a shared-memory-staged variant with the same order (below).
+#include <cstdlib>
+
 #include "common.cuh"
 #include "kernels.h"
 
@@ -101,15 +103,25 @@ __device__ __forceinline__ void cp_async16(void* dst, const void* src, bool vali
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(d), "l"(src), "r"(n) : "memory");
 }
 
+// With a token list, tile rows are the listed tokens (list[0 .. *n_list)),
+// and tiles past the list's end return at once.
 __global__ void __launch_bounds__(256, 1)
 gate_logits_tiled_kernel(const __nv_bfloat16* __restrict__ x, const __nv_bfloat16* __restrict__ wg,
-                         const float* __restrict__ bias, float* __restrict__ logits, int T, int H, int E) {
+                         const float* __restrict__ bias, float* __restrict__ logits, int T, int H, int E,
+                         const int32_t* __restrict__ list, const int32_t* __restrict__ n_list) {
     pdl_enter();
+    const int n_rows = list ? *n_list : T;
+    if ((int)blockIdx.x * kGT >= n_rows) return;
+    // token of tile row i (or -1 past the end)
+    auto token = [&](int i) -> int {
+        const int r = (int)blockIdx.x * kGT + i;
+        return r < n_rows ? (list ? list[r] : r) : -1;
+    };
     extern __shared__ __align__(16) uint8_t smem[];
     uint8_t* sx = smem;                                          // [stage][kGT][kSlab] bf16
     uint8_t* sw = smem + (size_t)kGStages * kGT * kSlab * 2;     // [stage][kGE][kSlab] bf16
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int t0 = blockIdx.x * kGT, e0 = blockIdx.y * kGE;
+    const int e0 = blockIdx.y * kGE;
     const int nslab = H / kSlab;
 
     auto load_slab = [&](int j) {
@@ -118,8 +130,8 @@ gate_logits_tiled_kernel(const __nv_bfloat16* __restrict__ x, const __nv_bfloat1
         for (int i = threadIdx.x; i < (kGT + kGE) * 32; i += 256) {
             const int row = i >> 5, c = i & 31;
             if (row < kGT) {
-                const int t = t0 + row;
-                const bool ok = t < T;
+                const int t = token(row);
+                const bool ok = t >= 0;
                 cp_async16(sx + (((size_t)st * kGT + row) * kSlab + 8 * c) * 2,
                            x + (size_t)(ok ? t : 0) * H + (size_t)j * kSlab + 8 * c, ok);
             } else {
@@ -190,8 +202,8 @@ gate_logits_tiled_kernel(const __nv_bfloat16* __restrict__ x, const __nv_bfloat1
     for (int a = 0; a < 8; ++a)
 #pragma unroll
         for (int b = 0; b < 8; ++b) {
-            const int t = t0 + tg + a, e = e0 + eg + b;
-            if (lane == ((a * 8 + b) & 31) && t < T && e < E) {
+            const int t = token(tg + a), e = e0 + eg + b;
+            if (lane == ((a * 8 + b) & 31) && t >= 0 && e < E) {
                 float l = acc[a][b];
                 if (bias) l = __fadd_rn(l, bias[e]);
                 logits[(size_t)t * E + e] = l;
@@ -253,76 +265,128 @@ __device__ __forceinline__ void warp_best(float& k, int& i) {
 constexpr int kSelWarps = 4;
 constexpr int kMaxE = 512;
 
-// One warp per token. Expert e lives in lane e % 32, slot e / 32.
+// Audit of router logits computed on the tensor cores (their fp32 sums run in
+// the hardware's own order, not the fixed order of the definition). Those
+// logits differ from the fixed-order ones by at most about
+// scale * ||x_t|| * ||w_e|| (|sum of the same products in two orders|), so an
+// expert choice whose every deciding comparison clears twice that bound is the
+// fixed-order choice; any other token is recomputed in the fixed order.
+struct GateAudit {
+    const __nv_bfloat16* x;   // [T, H]; null: logits are fixed-order already (no audit)
+    const float* wnorm_max;   // max_e ||wg[e]||_2 (one float)
+    float scale;              // bound on |tensor-core logit - fixed-order logit| / (||x_t|| * max ||w_e||)
+    int32_t* flagged;         // [T] tokens whose choice is too close to call (their logits are recomputed)
+    int32_t* n_flagged;       // their count
+};
+
+// One warp per token (every token, or those of `list` in grid-stride order).
+// Expert e lives in lane e % 32, slot e / 32.
 __global__ void __launch_bounds__(kSelWarps * 32)
 select_experts_kernel(const float* __restrict__ logits, const float* __restrict__ select_bias,
-                      int32_t* __restrict__ topk_ids, float* __restrict__ topk_w, RouteParams rp) {
+                      int32_t* __restrict__ topk_ids, float* __restrict__ topk_w, RouteParams rp, GateAudit au,
+                      const int32_t* __restrict__ list, const int32_t* __restrict__ n_list) {
     pdl_enter();
     __shared__ float s_key[kSelWarps][kMaxE];
     __shared__ float s_sig[kSelWarps][kMaxE];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int t = blockIdx.x * kSelWarps + warp;
-    if (t >= rp.T) return;
+    const int n_tok = list ? *n_list : rp.T;
+    for (int i = blockIdx.x * kSelWarps + warp; i < n_tok; i += gridDim.x * kSelWarps) {
+    const int t = list ? list[i] : i;
     const int E = rp.E, k = rp.top_k;
     const float* l = logits + (size_t)t * E;
     float* key = s_key[warp];
     float* sig = s_sig[warp];
     const bool sigmoid = rp.score == GBMOE_SIGMOID;
-    for (int e = lane; e < E; e += 32) {
-        float v = l[e];
-        if (sigmoid) {
-            float s = pinned_sigmoid(v);
-            sig[e] = s;
-            v = select_bias ? __fadd_rn(s, select_bias[e]) : s;
-        }
-        key[e] = choice_key(v);
-    }
-    __syncwarp();
-
-    // groups kept (bit g set); all experts allowed without group limiting
-    uint32_t kept = 0xffffffffu;
     const int G = sigmoid ? rp.n_group : 1;
-    if (G > 1) {
-        const int gs = E / G;
-        float gscore = -INFINITY;
-        if (lane < G) {
-            float a = -INFINITY, b = -INFINITY;  // two largest q of group `lane`
-            for (int e = lane * gs; e < (lane + 1) * gs; ++e) {
-                float v = key[e];
-                if (v > a) { b = a; a = v; } else if (v > b) { b = v; }
-            }
-            gscore = choice_key(__fadd_rn(a, b));  // inf + -inf is NaN
-        }
-        kept = 0u;
-        bool taken = false;
-        for (int r = 0; r < rp.topk_group; ++r) {
-            float kk = (lane < G && !taken) ? gscore : -INFINITY;
-            int ii = (lane < G && !taken) ? lane : kNone;
-            warp_best(kk, ii);
-            if (ii < 32) kept |= 1u << ii;  // always: topk_group <= G groups hold candidates
-            if (lane == ii) taken = true;
-        }
-    }
     const int gs = E / G;
-
-    // top-k over allowed experts, descending key, ties to the lower index
-    uint32_t used = 0u;  // bit s: expert lane + 32 s already chosen
     int sel_id = 0;
     float top_key = 0.0f;
-    for (int j = 0; j < k; ++j) {
-        float kk = -INFINITY;
-        int ii = kNone;
-        for (int s = 0, e = lane; e < E; ++s, e += 32) {
-            if ((used >> s) & 1u) continue;
-            if (!((kept >> (e / gs)) & 1u)) continue;
-            float v = key[e];
-            if (ii == kNone || better(v, e, kk, ii)) { kk = v; ii = e; }
+    {
+        for (int e = lane; e < E; e += 32) {
+            float v = l[e];
+            if (sigmoid) {
+                float s = pinned_sigmoid(v);
+                sig[e] = s;
+                v = select_bias ? __fadd_rn(s, select_bias[e]) : s;
+            }
+            key[e] = choice_key(v);
         }
-        warp_best(kk, ii);
-        // ii < E always (check_config keeps top_k within the kept groups' experts)
-        if (ii < E && (ii & 31) == lane) used |= 1u << (ii >> 5);
-        if (j == 0) top_key = kk;
-        if (lane == j) sel_id = ii < E ? ii : 0;
+        __syncwarp();
+
+        // groups kept (bit g set); all experts allowed without group limiting.
+        // margin_g: gap between the last kept and the best dropped group score
+        uint32_t kept = 0xffffffffu;
+        float margin_g = INFINITY;
+        if (G > 1) {
+            float gscore = -INFINITY;
+            if (lane < G) {
+                float a = -INFINITY, b = -INFINITY;  // two largest q of group `lane`
+                for (int e = lane * gs; e < (lane + 1) * gs; ++e) {
+                    float v = key[e];
+                    if (v > a) { b = a; a = v; } else if (v > b) { b = v; }
+                }
+                gscore = choice_key(__fadd_rn(a, b));  // inf + -inf is NaN
+            }
+            kept = 0u;
+            bool taken = false;
+            float last = 0.0f;
+            for (int r = 0; r <= rp.topk_group && r < G; ++r) {
+                float kk = (lane < G && !taken) ? gscore : -INFINITY;
+                int ii = (lane < G && !taken) ? lane : kNone;
+                warp_best(kk, ii);
+                if (r == rp.topk_group) {  // the best dropped group
+                    margin_g = last - kk;
+                    break;
+                }
+                if (ii < 32) kept |= 1u << ii;  // always: topk_group <= G groups hold candidates
+                if (lane == ii) taken = true;
+                last = kk;
+            }
+        }
+
+        // top-k over allowed experts, descending key, ties to the lower index;
+        // margin_k: smallest gap between consecutive keys of the k chosen and
+        // the best one left out
+        uint32_t used = 0u;  // bit s: expert lane + 32 s already chosen
+        float prev = 0.0f, margin_k = INFINITY;
+        for (int j = 0; j <= k; ++j) {
+            float kk = -INFINITY;
+            int ii = kNone;
+            for (int s = 0, e = lane; e < E; ++s, e += 32) {
+                if ((used >> s) & 1u) continue;
+                if (!((kept >> (e / gs)) & 1u)) continue;
+                float v = key[e];
+                if (ii == kNone || better(v, e, kk, ii)) { kk = v; ii = e; }
+            }
+            warp_best(kk, ii);
+            if (j > 0 && ii < E) margin_k = fminf(margin_k, prev - kk);
+            if (j == k) break;  // only the margin to the best expert left out
+            // ii < E always (check_config keeps top_k within the kept groups' experts)
+            if (ii < E && (ii & 31) == lane) used |= 1u << (ii >> 5);
+            if (j == 0) top_key = kk;
+            if (lane == j) sel_id = ii < E ? ii : 0;
+            prev = kk;
+        }
+
+        if (au.x) {
+        // bound on the logit error, and on the key error it causes (sigmoid:
+        // slope <= 1/4, plus a few units in the last place of the fp32 key)
+        float xx = 0.0f;
+        const __nv_bfloat16* xt = au.x + (size_t)t * rp.H;
+        for (int c = lane; c < rp.H / 8; c += 32) {
+            float xv[8];
+            Vec8<__nv_bfloat16>::load(xt + 8 * c, xv);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) xx = fmaf(xv[i], xv[i], xx);
+        }
+#pragma unroll
+        for (int d = 16; d >= 1; d >>= 1) xx += __shfl_xor_sync(0xffffffffu, xx, d);
+        // (plus a few units in the last place of the logits, for the bias add)
+        const float bl = au.scale * sqrtf(xx) * *au.wnorm_max + 1e-6f * (1.0f + fabsf(top_key));
+        const float bk = sigmoid ? 0.25f * bl + 1e-6f : bl;
+        const bool close = !(margin_k > 2.0f * bk) || !(margin_g > 4.0f * bk);
+        if (close && lane == 0) au.flagged[atomicAdd(au.n_flagged, 1)] = t;
+        }
     }
 
     // routing weights (lane j < k holds slot j)
@@ -354,27 +418,89 @@ select_experts_kernel(const float* __restrict__ logits, const float* __restrict_
         topk_ids[(size_t)t * k + lane] = sel_id;
         topk_w[(size_t)t * k + lane] = w;
     }
+    __syncwarp();
+    }
+}
+
+// max over experts of ||wg[e]||_2 (fp32) into *out: one CTA, a warp per row
+__global__ void __launch_bounds__(256)
+row_norm_max_kernel(const __nv_bfloat16* __restrict__ wg, int E, int H, float* __restrict__ out) {
+    pdl_enter();
+    __shared__ float s_max[8];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    float best = 0.0f;
+    for (int e = warp; e < E; e += 8) {
+        float ss = 0.0f;
+        for (int c = lane; c < H / 8; c += 32) {
+            float v[8];
+            Vec8<__nv_bfloat16>::load(wg + (size_t)e * H + 8 * c, v);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) ss = fmaf(v[i], v[i], ss);
+        }
+#pragma unroll
+        for (int d = 16; d >= 1; d >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, d);
+        best = fmaxf(best, sqrtf(ss));
+    }
+    if (lane == 0) s_max[warp] = best;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        float m = 0.0f;
+        for (int i = 0; i < 8; ++i) m = fmaxf(m, s_max[i]);
+        *out = m;
+    }
+}
+
+// Bound on |tensor-core logit - fixed-order logit| / (||x_t|| * max_e ||w_e||)
+// that the audit uses (from measured differences on the workloads, with a
+// safety factor; GBMOE_GATE_AUDIT_SCALE overrides it for tests).
+constexpr float kGateAuditScale = 2.0e-6f;
+
+static float gate_audit_scale() {
+    const char* v = std::getenv("GBMOE_GATE_AUDIT_SCALE");
+    if (!v || !*v) return kGateAuditScale;
+    char* end = nullptr;
+    const float f = std::strtof(v, &end);
+    return (end != v && *end == '\0' && f >= 0.0f) ? f : kGateAuditScale;
+}
+
+// shared-memory size of the tiled gate kernel, set once per device
+static cudaError_t gate_tiled_smem() {
+    static DeviceOnce smem_set;
+    return smem_set.run([] {
+        return cudaFuncSetAttribute(gate_logits_tiled_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)kGateTiledSmem);
+    });
 }
 
 cudaError_t launch_route(const RouteParams& rp, const void* x, const void* wg, const float* logit_bias,
                          const float* select_bias, float* logits, int32_t* topk_ids, float* topk_w,
-                         cudaStream_t stream) {
+                         const RouteScratch& rs, cudaStream_t stream) {
     if (rp.T == 0) return cudaSuccess;
     const int ey = (rp.E + kGateWarps * kGateExpertsPerWarp - 1) / (kGateWarps * kGateExpertsPerWarp);
     dim3 block(kGateWarps * 32);
-    if (rp.act_dtype == GBMOE_BF16) {
+    GateAudit au{};
+    if (rp.gate_tc) {
+        // tensor-core logits, then the audited choice
+        auto xp = static_cast<const __nv_bfloat16*>(x);
+        auto wp = static_cast<const __nv_bfloat16*>(wg);
+        if (const cudaError_t le = launch_k(row_norm_max_kernel, dim3(1), dim3(256), 0, stream, wp, rp.E, rp.H,
+                rs.audit); le != cudaSuccess)
+            return le;
+        if (cudaMemsetAsync(rs.audit + 1, 0, 4, stream) != cudaSuccess) return cudaErrorUnknown;
+        if (const cudaError_t le = launch_gate_tc(x, wg, logit_bias, logits, rp.T, rp.H, rp.E, rs.sched, rs.err,
+                stream); le != cudaSuccess)
+            return le;
+        au.x = xp; au.wnorm_max = rs.audit; au.scale = gate_audit_scale();
+        au.flagged = rs.flagged; au.n_flagged = reinterpret_cast<int32_t*>(rs.audit + 1);
+    } else if (rp.act_dtype == GBMOE_BF16) {
         auto xp = static_cast<const __nv_bfloat16*>(x);
         auto wp = static_cast<const __nv_bfloat16*>(wg);
         if (rp.T >= 1024) {
-            static DeviceOnce smem_set;
-            cudaError_t e = smem_set.run([] {
-                return cudaFuncSetAttribute(gate_logits_tiled_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                            (int)kGateTiledSmem);
-            });
-            if (e != cudaSuccess) return e;
+            if (const cudaError_t e = gate_tiled_smem(); e != cudaSuccess) return e;
             dim3 grid((rp.T + kGT - 1) / kGT, (rp.E + kGE - 1) / kGE);
             if (const cudaError_t le = launch_k(gate_logits_tiled_kernel, dim3(grid), dim3(256), kGateTiledSmem,
-                    stream, xp, wp, logit_bias, logits, rp.T, rp.H, rp.E); le != cudaSuccess)
+                    stream, xp, wp, logit_bias, logits, rp.T, rp.H, rp.E, static_cast<const int32_t*>(nullptr),
+                    static_cast<const int32_t*>(nullptr)); le != cudaSuccess)
                 return le;
         } else {
             dim3 grid((rp.T + 1) / 2, ey);
@@ -393,7 +519,24 @@ cudaError_t launch_route(const RouteParams& rp, const void* x, const void* wg, c
     cudaError_t err = cudaGetLastError();
     if (err != cudaSuccess) return err;
     if (const cudaError_t le = launch_k(select_experts_kernel, dim3((rp.T + kSelWarps - 1) / kSelWarps),
-            dim3(kSelWarps * 32), 0, stream, logits, select_bias, topk_ids, topk_w, rp); le != cudaSuccess)
+            dim3(kSelWarps * 32), 0, stream, logits, select_bias, topk_ids, topk_w, rp, au,
+            static_cast<const int32_t*>(nullptr), static_cast<const int32_t*>(nullptr)); le != cudaSuccess)
+        return le;
+    if ((err = cudaGetLastError()) != cudaSuccess || !rp.gate_tc) return err;
+    // flagged tokens: fixed-order logits, then their choice again (no audit)
+    const int32_t* n_flag = reinterpret_cast<const int32_t*>(rs.audit + 1);
+    if ((err = gate_tiled_smem()) != cudaSuccess) return err;
+    const dim3 lgrid((rp.T + kGT - 1) / kGT, (rp.E + kGE - 1) / kGE);  // tiles past the flagged count exit
+    if (const cudaError_t le = launch_k(gate_logits_tiled_kernel, lgrid, dim3(256), kGateTiledSmem, stream,
+            static_cast<const __nv_bfloat16*>(x), static_cast<const __nv_bfloat16*>(wg), logit_bias, logits, rp.T,
+            rp.H, rp.E, static_cast<const int32_t*>(rs.flagged), n_flag); le != cudaSuccess)
+        return le;
+    if ((err = cudaGetLastError()) != cudaSuccess) return err;
+    const int blocks = sm_count() * 4;
+    GateAudit none{};
+    if (const cudaError_t le = launch_k(select_experts_kernel, dim3(blocks), dim3(kSelWarps * 32), 0, stream, logits,
+            select_bias, topk_ids, topk_w, rp, none, static_cast<const int32_t*>(rs.flagged), n_flag);
+        le != cudaSuccess)
         return le;
     return cudaGetLastError();
 }

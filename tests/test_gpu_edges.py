@@ -175,3 +175,29 @@ def test_mxfp4_with_fp32_activations(route):
     ref = oracle.forward(wl, inp)
     assert np.array_equal(ids.cpu().numpy(), ref["topk_ids"])
     assert_close(act_np(out), ref["out"], 1e-5)
+
+
+@pytest.mark.parametrize("score", ["softmax", "sigmoid"])
+def test_tc_gate_audit_resolves_exact_ties(score):
+    """Integer router weights and activations make many logits tie exactly
+    (both orders sum them exactly): every such token is flagged by the audit,
+    recomputed in the fixed order, and chosen as the oracle chooses (ties to
+    the lower expert), on the tensor-core gate."""
+    T, H, E, k = 600, 512, 32, 4
+    rng = np.random.default_rng(8 if score == "softmax" else 9)
+    xi = rng.integers(-2, 3, size=(T, H)).astype(np.float32)
+    wi = rng.integers(-1, 2, size=(E, H)).astype(np.float32)
+    wi[E // 2:] = wi[: E // 2]  # duplicated router rows: exact ties in every token
+    extra = dict(score="sigmoid", n_group=4, topk_group=2) if score == "sigmoid" else {}
+    cfg = gb.make_config(T, H, 128, E, k, act="bf16", w="bf16", gate_route="tc", **extra)
+    x = torch.from_numpy(xi).cuda().to(torch.bfloat16)
+    wr = torch.from_numpy(wi).cuda().to(torch.bfloat16)
+    ws = workspace(cfg)
+    ids = torch.empty((T, k), dtype=torch.int32, device="cuda")
+    w = torch.empty((T, k), dtype=torch.float32, device="cuda")
+    gb.moe_route(cfg, x, wr, None, None, ids, w, ws)
+    torch.cuda.synchronize()
+    ref_ids, ref_w = oracle.route(oracle.gate_logits(xi, wi), k, score, True, extra.get("n_group", 1),
+                                  extra.get("topk_group", 1))
+    assert np.array_equal(ids.cpu().numpy(), ref_ids)
+    np.testing.assert_allclose(w.cpu().numpy(), ref_w, rtol=1e-5, atol=1e-7)
