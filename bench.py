@@ -316,7 +316,8 @@ def measure(args, wid: int, overrides, dist, world: int, rank: int, local: int, 
     shared, keep2 = wts(inp["shared"]) if wl.has_shared else (None, None)
     cfg = gb.make_config(wl.T, wl.H, wl.I, wl.E, wl.top_k, score=wl.score, renormalize=wl.renormalize,
                          n_group=wl.n_group, topk_group=wl.topk_group, routed_scale=wl.routed_scale, act=wl.act,
-                         w=wl.wq, has_shared=wl.has_shared, I_shared=wl.I_shared, ffn_route=args.route)
+                         w=wl.wq, has_shared=wl.has_shared, I_shared=wl.I_shared, ffn_route=args.route,
+                         gate_route=args.gate, combine_route=args.combine)
     ws = torch.empty(gb.workspace_size(cfg), dtype=torch.uint8, device=dev)
     out = torch.empty((wl.T, wl.H), dtype=x.dtype, device=dev)
     counts = torch.empty(wl.E, dtype=torch.int32, device=dev)
@@ -394,7 +395,7 @@ def measure(args, wid: int, overrides, dist, world: int, rank: int, local: int, 
               "simt": "moe_grouped_ffn, CUDA-core route"}[route]
     tpe = TRAFFIC_PER_ACTIVE_EXPERT.get((wl.name, route))
     extra = {"traffic": None if tpe is None else tpe * active, "kernel": kernel, "active_experts": active,
-             "route": route}
+             "route": route, "gate": gb.gate_route(cfg)}
     roofline = roofline_entry(routed_bytes, flops, ffn_ms, pk, pk_kind, extra)
 
     # end to end through the public host-buffer entry point
@@ -439,6 +440,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", type=int, default=2, help="synth.WORKLOADS id of the headline (2 = decode bf16)")
     ap.add_argument("--route", default="auto", choices=["auto", "stream", "simt", "tc", "tc_dequant", "tc_fp8"])
+    ap.add_argument("--gate", default="auto", choices=["auto", "simt", "tc"], help="router logits route")
+    ap.add_argument("--combine", default="auto", choices=["auto", "separate", "fused"], help="Weight Sum route")
     ap.add_argument("--ref-tokens", type=int, default=1, help="tokens per oracle step (reference arm)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-per-config", action="store_true",
@@ -476,7 +479,8 @@ def main():
     if head is None:  # --profile
         return
     per_config = {}
-    if not args.no_per_config and not args.set and args.route == "auto":
+    if not args.no_per_config and not args.set and args.route == "auto" and args.gate == "auto" \
+            and args.combine == "auto":
         for wid in PER_CONFIG:
             if wid == args.workload:
                 continue

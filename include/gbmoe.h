@@ -106,6 +106,18 @@ enum {
  * more, else SIMT. */
 enum { GBMOE_GATE_AUTO = 0, GBMOE_GATE_SIMT = 1, GBMOE_GATE_TC = 2 };
 
+/* Where moe_forward computes the Weight Sum. SEPARATE: moe_combine's gather
+ * kernel after the FFN. FUSED (tensor-core FFN routes GBMOE_FFN_TC and
+ * _TC_DEQUANT): in the down GEMM's epilogue, which writes topk_w * y of each
+ * pair into a slot buffer in pair order and counts, per token and 256 output
+ * columns, the slots written; the warp that writes the last one sums the
+ * token's slots in slot order (plus the shared expert's row, computed before
+ * the routed FFN) and writes out once: deterministic, no atomics on data.
+ * The slot is rounded to bf16 after the weight multiply (SEPARATE multiplies
+ * the bf16 row), so the two differ within rounding. Other FFN routes use
+ * SEPARATE. AUTO: SEPARATE (measured faster on GB300). */
+enum { GBMOE_COMBINE_AUTO = 0, GBMOE_COMBINE_SEPARATE = 1, GBMOE_COMBINE_FUSED = 2 };
+
 typedef struct gbmoe_config {
     int32_t T, H, I, E, top_k;
     int32_t score;        /* GBMOE_SOFTMAX or GBMOE_SIGMOID                         */
@@ -119,6 +131,7 @@ typedef struct gbmoe_config {
     int32_t I_shared;     /* its intermediate size                                  */
     int32_t ffn_route;    /* GBMOE_FFN_*                                            */
     int32_t gate_route;   /* GBMOE_GATE_*                                           */
+    int32_t combine_route; /* GBMOE_COMBINE_*                                       */
 } gbmoe_config;
 
 /* One set of expert weights (all experts stacked, E of them, or 1 for the

@@ -21,9 +21,11 @@ F32, BF16, FP8_E4M3_B128, INT4_G128, MXFP4 = 0, 1, 2, 3, 4
 SOFTMAX, SIGMOID = 0, 1
 FFN_AUTO, FFN_STREAM, FFN_SIMT, FFN_TC, FFN_TC_DEQUANT, FFN_TC_FP8 = 0, 1, 2, 3, 4, 5
 GATE_AUTO, GATE_SIMT, GATE_TC = 0, 1, 2
+COMBINE_AUTO, COMBINE_SEPARATE, COMBINE_FUSED = 0, 1, 2
 
 DTYPES = {"f32": F32, "bf16": BF16, "fp8_b128": FP8_E4M3_B128, "int4_g128": INT4_G128, "mxfp4": MXFP4}
 GATES = {"auto": GATE_AUTO, "simt": GATE_SIMT, "tc": GATE_TC}
+COMBINES = {"auto": COMBINE_AUTO, "separate": COMBINE_SEPARATE, "fused": COMBINE_FUSED}
 ROUTES = {"auto": FFN_AUTO, "stream": FFN_STREAM, "simt": FFN_SIMT, "tc": FFN_TC, "tc_dequant": FFN_TC_DEQUANT,
           "tc_fp8": FFN_TC_FP8}
 
@@ -46,7 +48,8 @@ class Config(ctypes.Structure):
                 ("top_k", ctypes.c_int32), ("score", ctypes.c_int32), ("renormalize", ctypes.c_int32),
                 ("n_group", ctypes.c_int32), ("topk_group", ctypes.c_int32), ("routed_scale", ctypes.c_float),
                 ("act_dtype", ctypes.c_int32), ("w_dtype", ctypes.c_int32), ("has_shared", ctypes.c_int32),
-                ("I_shared", ctypes.c_int32), ("ffn_route", ctypes.c_int32), ("gate_route", ctypes.c_int32)]
+                ("I_shared", ctypes.c_int32), ("ffn_route", ctypes.c_int32), ("gate_route", ctypes.c_int32),
+                ("combine_route", ctypes.c_int32)]
 
 
 class ExpertWeights(ctypes.Structure):
@@ -93,10 +96,10 @@ def status_string(status: int) -> str:
 
 def make_config(T, H, I, E, top_k, *, score="softmax", renormalize=True, n_group=1, topk_group=1,
                 routed_scale=1.0, act="bf16", w="bf16", has_shared=False, I_shared=0, ffn_route="auto",
-                gate_route="auto") -> Config:
+                gate_route="auto", combine_route="auto") -> Config:
     return Config(T, H, I, E, top_k, SOFTMAX if score == "softmax" else SIGMOID, int(bool(renormalize)), n_group,
                   topk_group, routed_scale, DTYPES[act], DTYPES[w], int(bool(has_shared)), I_shared,
-                  ROUTES[ffn_route], GATES[gate_route])
+                  ROUTES[ffn_route], GATES[gate_route], COMBINES[combine_route])
 
 
 def _ptr(t):

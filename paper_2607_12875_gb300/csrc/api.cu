@@ -35,6 +35,7 @@ int check_cfg(const gbmoe_config* c) {
     if (c->ffn_route < GBMOE_FFN_AUTO || c->ffn_route > GBMOE_FFN_TC_FP8) return GBMOE_EINVAL;
     if (c->gate_route < GBMOE_GATE_AUTO || c->gate_route > GBMOE_GATE_TC) return GBMOE_EINVAL;
     if (c->gate_route == GBMOE_GATE_TC && c->act_dtype != GBMOE_BF16) return GBMOE_EUNSUPPORTED;
+    if (c->combine_route < GBMOE_COMBINE_AUTO || c->combine_route > GBMOE_COMBINE_FUSED) return GBMOE_EINVAL;
     if (!std::isfinite(c->routed_scale)) return GBMOE_EINVAL;
     if (c->score == GBMOE_SIGMOID) {
         if (c->n_group < 1 || c->E % c->n_group != 0) return GBMOE_EINVAL;
@@ -89,7 +90,7 @@ size_t dequant_bytes(const gbmoe_config* c, int64_t n_rows, int E, int I) {
 }
 
 struct Layout {
-    size_t err, audit, flagged, logits, ids, w, counts, offsets, sorted, pos, perm, sched, h, xs, y, ysh, xin, xout, wdq,
+    size_t err, audit, flagged, arrive, logits, ids, w, counts, offsets, sorted, pos, perm, sched, h, xs, y, ysh, xin, xout, wdq,
         wdq_sh, aq, as, hq, hs, total;
 };
 
@@ -110,6 +111,7 @@ Layout layout(const gbmoe_config* c) {
     L.err = take(4);
     L.audit = take(8);
     L.flagged = take((size_t)T * 4);
+    L.arrive = take((size_t)T * (H / 256) * 4);
     L.logits = take((size_t)T * E * 4);
     L.ids = take((size_t)P * 4);
     L.w = take((size_t)P * 4);
@@ -409,15 +411,28 @@ int moe_forward(const gbmoe_config* cfg, const void* x, const void* w_router, co
     if ((s = cuda_status(launch_permute(ids, P, cfg->E, counts, offsets, sorted, pos, at<int32_t>(ws, L.perm), st))))
         return s;
     void* y = at<char>(ws, L.y);
-    FfnProblem pr = routed_problem(cfg, x, counts, offsets, sorted, experts, y, ws);
-    if ((s = run_ffn(cfg, pr, r_routed, st))) return s;
+    // the shared expert first: the routed down GEMM may fold the Weight Sum in
     void* ysh = nullptr;
     if (cfg->has_shared) {
         ysh = at<char>(ws, L.ysh);
         FfnProblem ps = shared_problem(cfg, x, shared, ysh, ws);
         if ((s = run_ffn(cfg, ps, r_shared, st))) return s;
     }
-    if ((s = cuda_status(launch_combine(y, w, pos, ysh, out, cfg->T, cfg->top_k, cfg->H, cfg->act_dtype, st))))
+    FfnProblem pr = routed_problem(cfg, x, counts, offsets, sorted, experts, y, ws);
+    const bool fused = cfg->combine_route == GBMOE_COMBINE_FUSED &&
+                       (r_routed == GBMOE_FFN_TC || r_routed == GBMOE_FFN_TC_DEQUANT);
+    if (fused) {  // Weight Sum in the down GEMM's epilogue
+        if (cudaMemsetAsync(at<int32_t>(ws, L.arrive), 0, (size_t)cfg->T * (cfg->H / 256) * 4, st) != cudaSuccess)
+            return GBMOE_ECUDA;
+        pr.fuse_k = cfg->top_k;
+        pr.topk_w = w;
+        pr.y_shared = ysh;
+        pr.out_final = out;
+        pr.arrive = at<int32_t>(ws, L.arrive);
+    }
+    if ((s = run_ffn(cfg, pr, r_routed, st))) return s;
+    if (!fused &&
+        (s = cuda_status(launch_combine(y, w, pos, ysh, out, cfg->T, cfg->top_k, cfg->H, cfg->act_dtype, st))))
         return s;
     if (topk_ids && cudaMemcpyAsync(topk_ids, ids, P * 4, cudaMemcpyDeviceToDevice, st) != cudaSuccess)
         return GBMOE_ECUDA;

@@ -112,6 +112,17 @@ struct Params {
     float* out_f32;
     const float* col_bias;
     int f32_cols;
+    // Weight Sum fused into the down GEMM (fuse_k > 0, the layer's top_k): row
+    // r is pair p = sorted_pair[r] = t*k + j; its output times topk_w[p] goes to
+    // slots[p] (pair order, bf16), and the thread completing the k-th arrival of
+    // token t on this N tile (arrive[t * n_tiles + nt]) sums the token's k
+    // slots in order j = 0..k-1, adds y_shared[t] and writes out_final[t].
+    int fuse_k;
+    const int32_t* sorted_pair;
+    const float* topk_w;
+    const __nv_bfloat16* y_shared;
+    __nv_bfloat16* out_final;
+    int32_t* arrive;
 };
 
 // Instruction descriptor, kind::f16: fp32 accumulator (bits 4-5 = 1), bf16 A
@@ -250,6 +261,53 @@ __device__ __forceinline__ Work decode_work(const Params& p, int w) {
 __device__ __forceinline__ void b_rows(const Params& p, const Work& wk, int& b0, int& b1) {
     b0 = wk.e * p.b_rows_per_expert + (p.swiglu ? wk.nt * (BN / 2) : wk.nt * BN);
     b1 = p.swiglu ? b0 : b0 + BN / 2;
+}
+
+// Weight Sum of the fused down GEMM, called by a whole epilogue warp after
+// its lanes stored their weighted slot rows (columns col0 .. col0 + BN of pair
+// `pair`, for the lanes with `valid`). Each such lane counts the arrival of
+// its token on this column range; the tokens whose k-th arrival this was are
+// then reduced by the whole warp, lane l taking 8 columns: the token's slots
+// in slot order (fp32, the same sum whichever warp does it), plus the shared
+// expert's row, rounded once; the counter is reset for the next call.
+__device__ __noinline__ void fused_weight_sum(const Params& p, bool valid, int64_t pair, int col0) {
+    const int lane = threadIdx.x & 31;
+    const int k = p.fuse_k;
+    const int64_t t = pair / k;
+    int32_t* cnt = p.arrive + t * p.n_tiles + col0 / BN;
+    bool last = false;
+    if (valid) {
+        __threadfence();  // the slot row is visible before the arrival is
+        last = atomicAdd(cnt, 1) == k - 1;
+    }
+    uint32_t done = __ballot_sync(0xffffffffu, last);
+    if (!done) return;
+    __threadfence();  // every slot row of those tokens is visible now
+    const int64_t H = p.out_cols;
+    while (done) {
+        const int src = __ffs(done) - 1;
+        done &= done - 1;
+        const int64_t tt = __shfl_sync(0xffffffffu, t, src);
+        if (lane == src) *cnt = 0;  // ready for the next call
+        for (int c = 8 * lane; c < BN; c += 256) {
+            float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+            for (int j = 0; j < k; ++j) {
+                // other SMs wrote these rows during this kernel: read them from L2
+                const uint4 u = __ldcg(reinterpret_cast<const uint4*>(p.out + (tt * k + j) * H + col0 + c));
+                const float v[8] = {bf16lo(u.x), bf16hi(u.x), bf16lo(u.y), bf16hi(u.y),
+                                    bf16lo(u.z), bf16hi(u.z), bf16lo(u.w), bf16hi(u.w)};
+#pragma unroll
+                for (int i = 0; i < 8; ++i) acc[i] = __fadd_rn(acc[i], v[i]);
+            }
+            if (p.y_shared) {
+                float v[8];
+                Vec8<__nv_bfloat16>::load(p.y_shared + tt * H + col0 + c, v);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) acc[i] = __fadd_rn(acc[i], v[i]);
+            }
+            Vec8<__nv_bfloat16>::store(p.out_final + tt * H + col0 + c, acc);
+        }
+    }
 }
 
 template <int WQ>
@@ -396,13 +454,21 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
             if (!warp_wait(&tfull[acc], acc_phase, abort_flag, p.err, p.wait_limit_ns)) break;
             tc_fence_after();
             const uint32_t t_row = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
-            const bool valid = r < wk.rows;
             // all 32 rows of this warp belong to the tile: one TMA store per 32 columns;
             // otherwise plain stores of the valid rows only (the rows past the tile's end
             // belong to the next expert and are written by another tile)
-            const bool via_tma = L::EPI_BYTES > 0 && q * 32 + 32 <= wk.rows && p.out_f32 == nullptr;
+            const bool via_tma = L::EPI_BYTES > 0 && q * 32 + 32 <= wk.rows && p.out_f32 == nullptr && p.fuse_k == 0;
             const int col0 = p.swiglu ? wk.nt * (BN / 2) : wk.nt * BN;
             __nv_bfloat16* dst = p.out + (wk.row0 + r) * (int64_t)p.out_cols + col0;
+            const bool valid = r < wk.rows;
+            // fused Weight Sum: this row's pair and routing weight; the row goes to its slot (pair order)
+            int64_t pair = 0;
+            float wpair = 0.0f;
+            if (p.fuse_k && valid) {
+                pair = p.sorted_pair[wk.row0 + r];
+                wpair = p.topk_w[pair];
+                dst = p.out + pair * (int64_t)p.out_cols + col0;
+            }
             const int ncols = p.swiglu ? BN / 2 : BN;
 #pragma unroll 1
             for (int c = 0; c < ncols; c += 32) {
@@ -431,11 +497,16 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
                         if (col < p.f32_cols) dst32[i] = p.col_bias ? __fadd_rn(v[i], p.col_bias[col]) : v[i];
                     }
                 } else if (valid) {
+                    if (p.fuse_k) {
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) v[i] *= wpair;
+                    }
                     store_bf16x32(dst + c, v);
                 }
             }
             tc_fence_before();
             mbar_arrive(&tempty[acc]);
+            if (p.fuse_k) fused_weight_sum(p, valid, pair, col0);  // warp-uniform
             if (++acc == 2) { acc = 0; acc_phase ^= 1; }
         }
         if (lane == 0) bulk_wait_all();  // stores complete before the CTA exits
@@ -754,6 +825,14 @@ cudaError_t launch_ffn_tc(const FfnProblem& pin, cudaStream_t stream) {
     d.K = p.I; d.n_tiles = p.H / BN; d.out_cols = p.H; d.b_rows_per_expert = p.H; d.swiglu = 0;
     d.out = static_cast<__nv_bfloat16*>(p.y);
     d.scale0 = p.s_down; d.scale1 = p.s_down;
+    if (p.fuse_k) {  // Weight Sum in the down GEMM: y holds the weighted slots (pair order)
+        d.fuse_k = p.fuse_k;
+        d.sorted_pair = p.sorted_pair;
+        d.topk_w = p.topk_w;
+        d.y_shared = static_cast<const __nv_bfloat16*>(p.y_shared);
+        d.out_final = static_cast<__nv_bfloat16*>(p.out_final);
+        d.arrive = p.arrive;
+    }
     return launch_gemm(p.w_dtype, mh, md, md, oy, d, max_m * d.n_tiles, stream);
 }
 

@@ -64,6 +64,15 @@ struct FfnProblem {
     float* h_s;                 //   and its 1x128 scales [n_rows, I/128]
     int32_t* sched;             // schedule ints, ffn_sched_ints(E, n_rows)
     int32_t* err;               // device error word
+    // Weight Sum fused into the down GEMM (tensor-core routes; fuse_k = top_k,
+    // 0 = off): y then receives topk_w[p] * y of pair p at row p (pair order)
+    // and out_final[t] = sum_j slots of t (+ y_shared[t]); arrive holds
+    // T * (H / 256) zeroed counters
+    int fuse_k;
+    const float* topk_w;
+    const void* y_shared;
+    void* out_final;
+    int32_t* arrive;
 };
 
 size_t ffn_sched_ints(int E, int64_t n_rows);

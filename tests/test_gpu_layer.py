@@ -188,3 +188,27 @@ def test_forward_is_deterministic():
     a, _, _ = _forward(wl, dev, "auto")
     b, _, _ = _forward(wl, dev, "auto")
     assert torch.equal(a, b)
+
+
+def test_fused_weight_sum_matches_oracle(wcase):
+    """The Weight Sum folded into the down GEMM's epilogue (tensor-core FFN
+    routes): every token against the oracle, deterministic over two calls, and
+    within rounding of the separate combine."""
+    wl, dev, ref = wcase["wl"], wcase["dev"], wcase["ref"]
+    route = gb.ffn_route(config(wl))
+    if route not in ("tc", "tc_dequant"):
+        pytest.skip("the fused Weight Sum runs on the bf16 tensor-core routes")
+    outs = []
+    for comb in ("fused", "fused", "separate"):
+        cfg = config(wl)
+        cfg.combine_route = gb.COMBINES[comb]
+        ws = workspace(cfg)
+        out = torch.empty((wl.T, wl.H), dtype=dev["x"].dtype, device="cuda")
+        gb.moe_forward(cfg, dev["x"], dev["w_router"], dev["logit_bias"], dev["select_bias"],
+                       wbundle(dev["experts"]), wbundle(dev["shared"]), out, ws)
+        torch.cuda.synchronize()
+        assert gb.moe_device_status(ws) == gb.OK
+        outs.append(out)
+    assert torch.equal(outs[0], outs[1])
+    assert_close(act_np(outs[0]), ref["out"], tol_for(wl), "fused Weight Sum")
+    assert_close(act_np(outs[0]), act_np(outs[2]), 2e-2, "fused vs separate")  # two bf16 roundings

@@ -161,3 +161,23 @@ def test_tc_fp8_route_with_shared_expert_and_timeout():
         del os.environ["GBMOE_TC_WAIT_LIMIT_NS"]
     out2, _ = forward(wl, dev, "tc_fp8")
     assert_close(act_np(out2), ref["out"], tol_for(wl))
+
+
+
+@pytest.mark.parametrize("wq", ["bf16", "int4_g128"])
+def test_fused_weight_sum_small_with_shared_expert(wq):
+    """Fused Weight Sum on a ragged problem with a shared expert (its row is
+    added by the warp that completes each token)."""
+    wl = BASE.replace(T=333, E=16, top_k=3, H=768, I=128, seed=211, wq=wq, has_shared=True, I_shared=256)
+    inp = synth.make_inputs(wl)
+    dev = to_device(wl, inp)
+    cfg = config(wl, "tc")
+    cfg.combine_route = gb.COMBINE_FUSED
+    ws = workspace(cfg)
+    out = torch.empty((wl.T, wl.H), dtype=torch.bfloat16, device="cuda")
+    gb.moe_forward(cfg, dev["x"], dev["w_router"], dev["logit_bias"], dev["select_bias"], wbundle(dev["experts"]),
+                   wbundle(dev["shared"]), out, ws)
+    torch.cuda.synchronize()
+    assert gb.moe_device_status(ws) == gb.OK
+    ref = oracle.forward(wl, inp)
+    assert_close(act_np(out), ref["out"], tol_for(wl))
