@@ -422,32 +422,26 @@ select_experts_kernel(const float* __restrict__ logits, const float* __restrict_
     }
 }
 
-// max over experts of ||wg[e]||_2 (fp32) into *out: one CTA, a warp per row
+// max over experts of ||wg[e]||_2 (fp32) into *out (zeroed beforehand): a
+// warp per router row; the maximum taken on the float bits, which order like
+// the values for non-negative floats
 __global__ void __launch_bounds__(256)
 row_norm_max_kernel(const __nv_bfloat16* __restrict__ wg, int E, int H, float* __restrict__ out) {
     pdl_enter();
-    __shared__ float s_max[8];
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    float best = 0.0f;
-    for (int e = warp; e < E; e += 8) {
-        float ss = 0.0f;
-        for (int c = lane; c < H / 8; c += 32) {
-            float v[8];
-            Vec8<__nv_bfloat16>::load(wg + (size_t)e * H + 8 * c, v);
+    const int lane = threadIdx.x & 31;
+    const int e = blockIdx.x * 8 + (threadIdx.x >> 5);
+    if (e >= E) return;
+    float ss = 0.0f;
+    for (int c = lane; c < H / 8; c += 32) {
+        float v[8];
+        Vec8<__nv_bfloat16>::load(wg + (size_t)e * H + 8 * c, v);
 #pragma unroll
-            for (int i = 0; i < 8; ++i) ss = fmaf(v[i], v[i], ss);
-        }
+        for (int i = 0; i < 8; ++i) ss = fmaf(v[i], v[i], ss);
+    }
 #pragma unroll
-        for (int d = 16; d >= 1; d >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, d);
-        best = fmaxf(best, sqrtf(ss));
-    }
-    if (lane == 0) s_max[warp] = best;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        float m = 0.0f;
-        for (int i = 0; i < 8; ++i) m = fmaxf(m, s_max[i]);
-        *out = m;
-    }
+    for (int d = 16; d >= 1; d >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, d);
+    if (lane == 0) atomicMax(reinterpret_cast<int*>(out), __float_as_int(sqrtf(ss)));
+}
 }
 
 // Bound on |tensor-core logit - fixed-order logit| / (||x_t|| * max_e ||w_e||)
@@ -483,10 +477,10 @@ cudaError_t launch_route(const RouteParams& rp, const void* x, const void* wg, c
         // tensor-core logits, then the audited choice
         auto xp = static_cast<const __nv_bfloat16*>(x);
         auto wp = static_cast<const __nv_bfloat16*>(wg);
-        if (const cudaError_t le = launch_k(row_norm_max_kernel, dim3(1), dim3(256), 0, stream, wp, rp.E, rp.H,
-                rs.audit); le != cudaSuccess)
+        if (cudaMemsetAsync(rs.audit, 0, 8, stream) != cudaSuccess) return cudaErrorUnknown;  // norm max, count
+        if (const cudaError_t le = launch_k(row_norm_max_kernel, dim3((rp.E + 7) / 8), dim3(256), 0, stream, wp,
+                rp.E, rp.H, rs.audit); le != cudaSuccess)
             return le;
-        if (cudaMemsetAsync(rs.audit + 1, 0, 4, stream) != cudaSuccess) return cudaErrorUnknown;
         if (const cudaError_t le = launch_gate_tc(x, wg, logit_bias, logits, rp.T, rp.H, rp.E, rs.sched, rs.err,
                 stream); le != cudaSuccess)
             return le;
