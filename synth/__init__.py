@@ -138,8 +138,8 @@ class Workload:
         return dataclasses.replace(self, **kw)
 
 
-# The five layer shapes of the benchmark grid. Seeds 0 and 3 are given by the
-# workload descriptions; 1, 2 and 4 are chosen here.
+# The six layer shapes of the benchmark grid. Seeds 0 and 3 are given by the
+# workload descriptions; 1, 2, 4 and 5 are chosen here.
 WORKLOADS = {
     1: Workload("tiny_f32_T64_H256_E8_k2_I512", 64, 256, 512, 8, 2, "f32", "f32", seed=0),
     2: Workload("decode_bf16_T32_H4096_E128_k8_I1536", 32, 4096, 1536, 128, 8, "bf16", "bf16", seed=1),
