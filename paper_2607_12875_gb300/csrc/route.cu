@@ -442,7 +442,6 @@ row_norm_max_kernel(const __nv_bfloat16* __restrict__ wg, int E, int H, float* _
     for (int d = 16; d >= 1; d >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, d);
     if (lane == 0) atomicMax(reinterpret_cast<int*>(out), __float_as_int(sqrtf(ss)));
 }
-}
 
 // Bound on |tensor-core logit - fixed-order logit| / (||x_t|| * max_e ||w_e||)
 // that the audit uses (from measured differences on the workloads, with a
