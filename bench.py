@@ -266,7 +266,8 @@ def launches_per_step(wl, route: str, shared_route) -> int:
     def ffn(r, routed):
         if r == "tc_fp8":  # schedule, x quantisation, gate/up GEMM, h quantisation, down GEMM
             return 5
-        return 3 + (1 if routed and r in ("tc", "tc_dequant") else 0) + (3 if r == "tc_dequant" else 0)
+        gemm = r in ("tc", "tc_dequant", "tc_pair", "tc_pair_dequant")
+        return 3 + (1 if routed and gemm else 0) + (3 if r in ("tc_dequant", "tc_pair_dequant") else 0)
 
     n = 2 + (1 if wl.P <= 1024 else 3) + ffn(route, True) + 1
     if shared_route is not None:
@@ -404,6 +405,10 @@ def measure(args, wid: int, overrides, dist, world: int, rank: int, local: int, 
                             "gate/up GEMM with SwiGLU + down GEMM)",
               "tc_fp8": "moe_grouped_ffn, fp8 tcgen05 route (two-term e4m3 quantisation of the rows + gate/up "
                         "GEMM with per-k-block promotion and SwiGLU + quantisation of h + down GEMM)",
+              "tc_pair": "moe_grouped_ffn, tcgen05 CTA-pair route (row gather + gate/up GEMM with SwiGLU + down "
+                         "GEMM, cta_group::2 MMAs of 256 rows)",
+              "tc_pair_dequant": "moe_grouped_ffn, tcgen05 CTA-pair decode-once route (3 weight-decode passes + "
+                                 "row gather + gate/up GEMM with SwiGLU + down GEMM, cta_group::2 MMAs)",
               "simt": "moe_grouped_ffn, CUDA-core route"}[route]
     tpe = TRAFFIC_PER_ACTIVE_EXPERT.get((wl.name, route))
     extra = {"traffic": None if tpe is None else tpe * active, "kernel": kernel, "active_experts": active,
@@ -451,7 +456,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", type=int, default=2, help="synth.WORKLOADS id of the headline (2 = decode bf16)")
-    ap.add_argument("--route", default="auto", choices=["auto", "stream", "simt", "tc", "tc_dequant", "tc_fp8"])
+    ap.add_argument("--route", default="auto", choices=["auto", "stream", "simt", "tc", "tc_dequant", "tc_fp8", "tc_pair", "tc_pair_dequant"])
     ap.add_argument("--gate", default="auto", choices=["auto", "simt", "tc"], help="router logits route")
     ap.add_argument("--combine", default="auto", choices=["auto", "separate", "fused"], help="Weight Sum route")
     ap.add_argument("--ref-tokens", type=int, default=1, help="tokens per oracle step (reference arm)")

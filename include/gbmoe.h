@@ -79,15 +79,24 @@ enum { GBMOE_SOFTMAX = 0, GBMOE_SIGMOID = 1 };
  * more rows per expert (several M tiles reuse each weight tile) AUTO takes
  * GBMOE_FFN_TC_DEQUANT: one pass decodes the active experts' weights to a
  * bf16 copy in the workspace (the same bf16 values the in-GEMM decode makes),
- * then the bf16 GEMM runs on it. */
+ * then the bf16 GEMM runs on it. The _PAIR routes run the same GEMM on CTA
+ * pairs (tcgen05 cta_group::2): one MMA of 256 rows per pair, each CTA
+ * holding 128 rows of A and half of the bf16 weight tile, which halves the
+ * weight bytes each SM reads per MMA; an expert's rows are then covered in
+ * 256-row tiles, so AUTO takes them only from P/E >= 1024 (little padding).
+ * Their outputs equal the one-CTA routes' bit for bit. TC_PAIR needs bf16
+ * weights; quantised weights take TC_PAIR_DEQUANT. */
 enum {
     GBMOE_FFN_AUTO = 0,
     GBMOE_FFN_STREAM = 1,     /* weight streaming: few rows per expert (decode)       */
     GBMOE_FFN_SIMT = 2,       /* CUDA-core tiled GEMM (fp32 activations, any weights) */
     GBMOE_FFN_TC = 3,         /* tcgen05/TMEM/TMA grouped GEMM (bf16 activations)     */
     GBMOE_FFN_TC_DEQUANT = 4, /* as TC, quantised weights decoded once beforehand     */
-    GBMOE_FFN_TC_FP8 = 5      /* fp8 tensor cores: FP8_E4M3_B128 weights as stored,
+    GBMOE_FFN_TC_FP8 = 5,     /* fp8 tensor cores: FP8_E4M3_B128 weights as stored,
                                  activations quantised to e4m3 per 1x128 block      */
+    GBMOE_FFN_TC_PAIR = 6,    /* as TC on CTA pairs: one MMA of 256 rows per pair
+                                 (each CTA holds and decodes half the weight tile)  */
+    GBMOE_FFN_TC_PAIR_DEQUANT = 7 /* as TC_DEQUANT, the bf16 GEMM on CTA pairs      */
 };
 
 /* How the MoE Gate computes the router logits. SIMT: CUDA cores in the fixed
@@ -107,8 +116,8 @@ enum {
 enum { GBMOE_GATE_AUTO = 0, GBMOE_GATE_SIMT = 1, GBMOE_GATE_TC = 2 };
 
 /* Where moe_forward computes the Weight Sum. SEPARATE: moe_combine's gather
- * kernel after the FFN. FUSED (tensor-core FFN routes GBMOE_FFN_TC and
- * _TC_DEQUANT): in the down GEMM's epilogue, which writes topk_w * y of each
+ * kernel after the FFN. FUSED (tensor-core FFN routes GBMOE_FFN_TC,
+ * _TC_DEQUANT, _TC_PAIR and _TC_PAIR_DEQUANT): in the down GEMM's epilogue, which writes topk_w * y of each
  * pair into a slot buffer in pair order and counts, per token and 256 output
  * columns, the slots written; the warp that writes the last one sums the
  * token's slots in slot order (plus the shared expert's row, computed before
@@ -170,7 +179,7 @@ int gbmoe_check_config(const gbmoe_config* cfg);
  * other calls need no more). 0 if the config is invalid. */
 size_t gbmoe_workspace_size(const gbmoe_config* cfg);
 
-/* The FFN route (GBMOE_FFN_STREAM, _SIMT, _TC or _TC_DEQUANT) that moe_forward runs for
+/* The FFN route (one of GBMOE_FFN_STREAM .. _TC_PAIR_DEQUANT) that moe_forward runs for
  * cfg: for the routed experts (shared = 0) or the shared expert (shared = 1).
  * Negative status if the config is invalid. */
 int gbmoe_ffn_route(const gbmoe_config* cfg, int shared);
@@ -278,8 +287,8 @@ int moe_forward_hostio(const gbmoe_config* cfg, const void* x_host, const void* 
  * Reads (and clears) the device error word that bounded device-side waits
  * set in `workspace`, after synchronising `stream`. *status receives GBMOE_OK
  * or GBMOE_EDEVICE_TIMEOUT. This is the only call that synchronises.
- * The waits are those of the tensor-core FFN kernels (GBMOE_FFN_TC and
- * _TC_DEQUANT): each gives up after 2 s, stops issuing work, lets the copies
+ * The waits are those of the tensor-core FFN kernels (the GBMOE_FFN_TC*
+ * routes): each gives up after 2 s, stops issuing work, lets the copies
  * and MMAs it issued finish, and sets the word; the call's outputs are then
  * incomplete. For tests of this path the environment variable
  * GBMOE_TC_WAIT_LIMIT_NS (read at every call) lowers the limit, in ns.

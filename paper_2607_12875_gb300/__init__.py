@@ -19,7 +19,7 @@ LIB_PATH = os.path.join(_HERE, "libgbmoe.so")
 OK, EINVAL, EUNSUPPORTED, EWORKSPACE, ECUDA, EDEVICE_TIMEOUT = 0, -1, -2, -3, -4, -5
 F32, BF16, FP8_E4M3_B128, INT4_G128, MXFP4 = 0, 1, 2, 3, 4
 SOFTMAX, SIGMOID = 0, 1
-FFN_AUTO, FFN_STREAM, FFN_SIMT, FFN_TC, FFN_TC_DEQUANT, FFN_TC_FP8 = 0, 1, 2, 3, 4, 5
+FFN_AUTO, FFN_STREAM, FFN_SIMT, FFN_TC, FFN_TC_DEQUANT, FFN_TC_FP8, FFN_TC_PAIR, FFN_TC_PAIR_DEQUANT = range(8)
 GATE_AUTO, GATE_SIMT, GATE_TC = 0, 1, 2
 COMBINE_AUTO, COMBINE_SEPARATE, COMBINE_FUSED = 0, 1, 2
 
@@ -27,7 +27,7 @@ DTYPES = {"f32": F32, "bf16": BF16, "fp8_b128": FP8_E4M3_B128, "int4_g128": INT4
 GATES = {"auto": GATE_AUTO, "simt": GATE_SIMT, "tc": GATE_TC}
 COMBINES = {"auto": COMBINE_AUTO, "separate": COMBINE_SEPARATE, "fused": COMBINE_FUSED}
 ROUTES = {"auto": FFN_AUTO, "stream": FFN_STREAM, "simt": FFN_SIMT, "tc": FFN_TC, "tc_dequant": FFN_TC_DEQUANT,
-          "tc_fp8": FFN_TC_FP8}
+          "tc_fp8": FFN_TC_FP8, "tc_pair": FFN_TC_PAIR, "tc_pair_dequant": FFN_TC_PAIR_DEQUANT}
 
 # every function include/gbmoe.h declares
 EXPORTS = ("gbmoe_status_string", "gbmoe_check_config", "gbmoe_workspace_size", "gbmoe_ffn_route",

@@ -20,6 +20,12 @@ size_t align_up(size_t v) { return (v + kAlign - 1) & ~(kAlign - 1); }
 size_t act_bytes(int act) { return act == GBMOE_F32 ? 4 : 2; }
 
 bool quantised_weights(int w) { return w == GBMOE_FP8_E4M3_B128 || w == GBMOE_INT4_G128 || w == GBMOE_MXFP4; }
+// routes that run the bf16-operand tensor-core GEMM (launch_ffn_tc)
+bool bf16_gemm_route(int r) {
+    return r == GBMOE_FFN_TC || r == GBMOE_FFN_TC_DEQUANT || r == GBMOE_FFN_TC_PAIR || r == GBMOE_FFN_TC_PAIR_DEQUANT;
+}
+bool pair_route(int r) { return r == GBMOE_FFN_TC_PAIR || r == GBMOE_FFN_TC_PAIR_DEQUANT; }
+bool dequant_route(int r) { return r == GBMOE_FFN_TC_DEQUANT || r == GBMOE_FFN_TC_PAIR_DEQUANT; }
 
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
@@ -32,7 +38,7 @@ int check_cfg(const gbmoe_config* c) {
     if (c->w_dtype < GBMOE_F32 || c->w_dtype > GBMOE_MXFP4) return GBMOE_EINVAL;
     if (c->has_shared != 0 && c->has_shared != 1) return GBMOE_EINVAL;
     if (c->has_shared && c->I_shared <= 0) return GBMOE_EINVAL;
-    if (c->ffn_route < GBMOE_FFN_AUTO || c->ffn_route > GBMOE_FFN_TC_FP8) return GBMOE_EINVAL;
+    if (c->ffn_route < GBMOE_FFN_AUTO || c->ffn_route > GBMOE_FFN_TC_PAIR_DEQUANT) return GBMOE_EINVAL;
     if (c->gate_route < GBMOE_GATE_AUTO || c->gate_route > GBMOE_GATE_TC) return GBMOE_EINVAL;
     if (c->gate_route == GBMOE_GATE_TC && c->act_dtype != GBMOE_BF16) return GBMOE_EUNSUPPORTED;
     if (c->combine_route < GBMOE_COMBINE_AUTO || c->combine_route > GBMOE_COMBINE_FUSED) return GBMOE_EINVAL;
@@ -50,8 +56,7 @@ int check_cfg(const gbmoe_config* c) {
     if (c->score == GBMOE_SIGMOID && c->n_group > 32) return GBMOE_EUNSUPPORTED;
     if ((int64_t)c->T * c->top_k > (int64_t(1) << 30)) return GBMOE_EUNSUPPORTED;
     if (c->act_dtype == GBMOE_BF16 && c->w_dtype == GBMOE_F32) return GBMOE_EUNSUPPORTED;
-    if ((c->ffn_route == GBMOE_FFN_TC || c->ffn_route == GBMOE_FFN_TC_DEQUANT) && c->act_dtype != GBMOE_BF16)
-        return GBMOE_EUNSUPPORTED;
+    if (bf16_gemm_route(c->ffn_route) && c->act_dtype != GBMOE_BF16) return GBMOE_EUNSUPPORTED;
     if (c->ffn_route == GBMOE_FFN_TC_FP8 && (c->act_dtype != GBMOE_BF16 || c->w_dtype != GBMOE_FP8_E4M3_B128))
         return GBMOE_EUNSUPPORTED;
     return GBMOE_OK;
@@ -75,8 +80,13 @@ int pick_route(const gbmoe_config* c, int64_t n_rows, int E, int I) {
         // activation codes keep bf16-level accuracy)
         if (ffn_tc_fp8_supported(probe)) return GBMOE_FFN_TC_FP8;
         if (ffn_tc_supported(probe)) {
-            return quantised_weights(c->w_dtype) && n_rows >= kDequantRowsPerExpert * E ? GBMOE_FFN_TC_DEQUANT
-                                                                                        : GBMOE_FFN_TC;
+            const bool dequant = quantised_weights(c->w_dtype) && n_rows >= kDequantRowsPerExpert * E;
+            // CTA pairs (256-row tiles) once experts are deep enough that the
+            // padding of their last tile stays small; they multiply bf16 tiles
+            if (dequant) probe.w_dq = &probe;
+            const bool pairs = n_rows >= kPairRowsPerExpert * E && ffn_tc_pair_supported(probe);
+            if (dequant) return pairs ? GBMOE_FFN_TC_PAIR_DEQUANT : GBMOE_FFN_TC_DEQUANT;
+            return pairs && c->w_dtype == GBMOE_BF16 ? GBMOE_FFN_TC_PAIR : GBMOE_FFN_TC;
         }
     }
     return GBMOE_FFN_SIMT;
@@ -85,7 +95,7 @@ int pick_route(const gbmoe_config* c, int64_t n_rows, int E, int I) {
 // Bytes of the bf16 weight copy the TC_DEQUANT route decodes into (0 when
 // the route of that problem does not use one).
 size_t dequant_bytes(const gbmoe_config* c, int64_t n_rows, int E, int I) {
-    if (!quantised_weights(c->w_dtype) || pick_route(c, n_rows, E, I) != GBMOE_FFN_TC_DEQUANT) return 0;
+    if (!quantised_weights(c->w_dtype) || !dequant_route(pick_route(c, n_rows, E, I))) return 0;
     return (size_t)3 * E * c->H * I * 2;
 }
 
@@ -200,13 +210,19 @@ int route_launchable(const gbmoe_config* c, int route, int I) {
         case GBMOE_FFN_SIMT: return GBMOE_OK;
         case GBMOE_FFN_TC:
         case GBMOE_FFN_TC_DEQUANT:
-        case GBMOE_FFN_TC_FP8: {
+        case GBMOE_FFN_TC_FP8:
+        case GBMOE_FFN_TC_PAIR:
+        case GBMOE_FFN_TC_PAIR_DEQUANT: {
             FfnProblem probe{};
             probe.act_dtype = c->act_dtype;
             probe.w_dtype = c->w_dtype;
             probe.H = c->H;
             probe.I = I;
-            const bool ok = route == GBMOE_FFN_TC_FP8 ? ffn_tc_fp8_supported(probe) : ffn_tc_supported(probe);
+            // the decode-once routes run the bf16 kernel (a non-null w_dq says so)
+            if (route == GBMOE_FFN_TC_PAIR_DEQUANT && quantised_weights(c->w_dtype)) probe.w_dq = &probe;
+            const bool ok = route == GBMOE_FFN_TC_FP8   ? ffn_tc_fp8_supported(probe)
+                            : pair_route(route) ? ffn_tc_pair_supported(probe)
+                                                : ffn_tc_supported(probe);
             return ok ? GBMOE_OK : GBMOE_EUNSUPPORTED;
         }
         default: return GBMOE_EINVAL;
@@ -220,7 +236,10 @@ int run_ffn(const gbmoe_config* c, FfnProblem& p, int route, cudaStream_t stream
         case GBMOE_FFN_STREAM: err = launch_ffn_stream(p, stream); break;
         case GBMOE_FFN_SIMT: err = launch_ffn_simt(p, stream); break;
         case GBMOE_FFN_TC_FP8: err = launch_ffn_tc_fp8(p, stream); break;
-        default: err = launch_ffn_tc(p, stream); break;  // GBMOE_FFN_TC, GBMOE_FFN_TC_DEQUANT
+        default:  // GBMOE_FFN_TC, _TC_DEQUANT, _TC_PAIR, _TC_PAIR_DEQUANT
+            p.cta_pair = pair_route(route) ? 1 : 0;
+            err = launch_ffn_tc(p, stream);
+            break;
     }
     return cuda_status(err);
 }
@@ -420,7 +439,7 @@ int moe_forward(const gbmoe_config* cfg, const void* x, const void* w_router, co
     }
     FfnProblem pr = routed_problem(cfg, x, counts, offsets, sorted, experts, y, ws);
     const bool fused = cfg->combine_route == GBMOE_COMBINE_FUSED &&
-                       (r_routed == GBMOE_FFN_TC || r_routed == GBMOE_FFN_TC_DEQUANT);
+                       bf16_gemm_route(r_routed);
     if (fused) {  // Weight Sum in the down GEMM's epilogue
         if (cudaMemsetAsync(at<int32_t>(ws, L.arrive), 0, (size_t)cfg->T * (cfg->H / 256) * 4, st) != cudaSuccess)
             return GBMOE_ECUDA;

@@ -48,40 +48,55 @@ namespace tc {
 
 constexpr int BM = 128, BN = 256, BK = 64;  // BK bf16 = 128 bytes = one swizzle row
 constexpr int A_BYTES = BM * BK * 2;
-constexpr int B_BYTES = BN * BK * 2;
+constexpr int B_BYTES = BN * BK * 2;  // bf16 B tile of one MMA (a CTA of a pair holds half)
 constexpr int TMEM_COLS = 512;
-constexpr int CONVERT_WARPS = 8;  // one thread per B row (BN = 256)
 constexpr int kFp8PrefetchAhead = 4;  // k-blocks the fp8 producer prefetches into L2 ahead of its loads
 
-// Per weight format: bytes of the raw B tile TMA brings in (0 = B is loaded
-// as bf16 directly), pipeline depth, threads.
+// Bytes of the raw weight tile (BN rows x BK elements) TMA brings in; 0: B is
+// loaded as bf16 directly.
 template <int WQ>
 struct Fmt;
 template <>
 struct Fmt<GBMOE_BF16> {
-    static constexpr int RAW_BYTES = 0, STAGES = 4, THREADS = 192;
+    static constexpr int RAW_BYTES = 0;
 };
 template <>
 struct Fmt<GBMOE_FP8_E4M3_B128> {
-    static constexpr int RAW_BYTES = BN * BK, STAGES = 3, THREADS = 192 + CONVERT_WARPS * 32;
+    static constexpr int RAW_BYTES = BN * BK;
 };
 template <>
 struct Fmt<GBMOE_INT4_G128> {
-    static constexpr int RAW_BYTES = BN * BK / 2, STAGES = 4, THREADS = 192 + CONVERT_WARPS * 32;
+    static constexpr int RAW_BYTES = BN * BK / 2;
 };
 template <>
 struct Fmt<GBMOE_MXFP4> {
-    static constexpr int RAW_BYTES = BN * BK / 2, STAGES = 4, THREADS = 192 + CONVERT_WARPS * 32;
+    static constexpr int RAW_BYTES = BN * BK / 2;
 };
 
 // nibble-packed formats: a raw row of BK elements is BK / 2 bytes
 template <int WQ>
 constexpr bool packed4() { return WQ == GBMOE_INT4_G128 || WQ == GBMOE_MXFP4; }
 
-template <int WQ>
+// Per weight format WQ and CTA group CG: CG = 1, one CTA per 128 x 256 tile;
+// CG = 2, a CTA pair per 256 x 256 tile, each CTA holding 128 A rows and 128
+// of the 256 B rows (bf16 B only: quantised weights are decoded beforehand
+// for pairs). Pipeline depth as shared memory allows.
+template <int WQ, int CG>
+struct Cfg {
+    static_assert(CG == 1 || WQ == GBMOE_BF16, "CTA pairs take bf16 B tiles");
+    static constexpr int RAW = Fmt<WQ>::RAW_BYTES / CG;  // raw B bytes per stage of one CTA
+    static constexpr int B_HELD = B_BYTES / CG;          // bf16 B bytes per stage of one CTA
+    static constexpr int B_ROWS = BN / CG;               // B rows of one CTA
+    static constexpr int CONVERT_WARPS = RAW ? B_ROWS / 32 : 0;  // one thread per B row
+    static constexpr int THREADS = 192 + CONVERT_WARPS * 32;
+    static constexpr int STAGES = CG == 1 ? (WQ == GBMOE_FP8_E4M3_B128 ? 3 : 4) : (RAW ? 5 : 6);
+};
+
+template <int WQ, int CG>
 struct Layout {
-    static constexpr int STAGES = Fmt<WQ>::STAGES;
-    static constexpr int STAGE_BYTES = A_BYTES + B_BYTES + Fmt<WQ>::RAW_BYTES;
+    using C = Cfg<WQ, CG>;
+    static constexpr int STAGES = C::STAGES;
+    static constexpr int STAGE_BYTES = A_BYTES + C::B_HELD + C::RAW;
     static constexpr int NUM_BARS = 3 * STAGES + 4 + 1;
     static constexpr int BASE_BYTES = 1024 + STAGES * STAGE_BYTES + NUM_BARS * 8 + 16;
     // output staging for TMA stores: 4 epilogue warps x 2 buffers x (32 rows x 64 bytes),
@@ -126,17 +141,59 @@ struct Params {
 };
 
 // Instruction descriptor, kind::f16: fp32 accumulator (bits 4-5 = 1), bf16 A
-// and B (bits 7-9, 10-12 = 1), both K-major, N/8 in bits 17-22, M/16 in 24-28.
+// and B (bits 7-9, 10-12 = 1), both K-major, N/8 in bits 17-22, M/16 in 24-28
+// (M = 128 per CTA, 256 for a CTA pair).
+template <int CG>
 constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
-                            ((uint32_t)(BM >> 4) << 24);
+                            ((uint32_t)((BM * CG) >> 4) << 24);
 
+template <int CG>
 __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t accumulate) {
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-        "l"(a_desc), "l"(b_desc), "r"(kIdesc), "r"(accumulate)
-        : "memory");
+    if constexpr (CG == 1)
+        asm volatile(
+            "{\n\t.reg .pred p;\n\t"
+            "setp.ne.b32 p, %4, 0;\n\t"
+            "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+            "l"(a_desc), "l"(b_desc), "r"(kIdesc<1>), "r"(accumulate)
+            : "memory");
+    else
+        asm volatile(
+            "{\n\t.reg .pred p;\n\t"
+            "setp.ne.b32 p, %4, 0;\n\t"
+            "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+            "l"(a_desc), "l"(b_desc), "r"(kIdesc<2>), "r"(accumulate)
+            : "memory");
+}
+
+// completion of the MMAs issued so far -> one arrival on `bar` (CG = 2: on
+// the barrier at the same offset in each CTA of cta_mask)
+template <int CG>
+__device__ __forceinline__ void commit_to(uint64_t* bar, uint16_t cta_mask) {
+    if constexpr (CG == 1) mma_commit(bar);
+    else mma_commit_pair(bar, cta_mask);
+}
+
+template <int CG>
+__device__ __forceinline__ void tmem_alloc(uint32_t* slot) {
+    if constexpr (CG == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(slot)),
+                     "r"(TMEM_COLS)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    } else {
+        asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(slot)),
+                     "r"(TMEM_COLS)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+    }
+}
+
+template <int CG>
+__device__ __forceinline__ void tmem_dealloc(uint32_t base) {
+    if constexpr (CG == 1)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(base), "r"(TMEM_COLS) : "memory");
+    else
+        asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(base), "r"(TMEM_COLS) : "memory");
 }
 
 // 32 fp32 -> 32 bf16 into row `lane` of a 32-row x 64-byte staging buffer in
@@ -239,11 +296,14 @@ __device__ __forceinline__ __nv_bfloat162 e8m0_bf16x2(uint32_t s) {
 
 struct Work {
     int e, m, nt;
-    int64_t row0;  // absolute first row of the M tile
-    int rows;      // valid rows in the tile
+    int64_t row0;  // absolute first row of this CTA's 128 rows of the M tile
+    int rows;      // valid rows among them (<= 0: none)
 };
 
-__device__ __forceinline__ Work decode_work(const Params& p, int w) {
+// Work item w: M tile w / n_tiles of the list (BM * CG rows of one expert),
+// N tile w % n_tiles; CTA `rank` of a pair takes the tile's rows rank*BM ..
+template <int CG>
+__device__ __forceinline__ Work decode_work(const Params& p, int w, uint32_t rank) {
     const int2* tiles = reinterpret_cast<const int2*>(p.sched + sched_tiles_offset(p.E));
     const int mt = w / p.n_tiles;
     Work r;
@@ -252,8 +312,9 @@ __device__ __forceinline__ Work decode_work(const Params& p, int w) {
     r.e = t.x;
     r.m = t.y;
     const int64_t cnt = p.counts ? p.counts[r.e] : p.n_rows;
-    r.row0 = (p.offsets ? p.offsets[r.e] : 0) + (int64_t)r.m * BM;
-    r.rows = (int)min64(BM, cnt - (int64_t)r.m * BM);
+    const int64_t first = (int64_t)r.m * (BM * CG) + (int64_t)rank * BM;
+    r.row0 = (p.offsets ? p.offsets[r.e] : 0) + first;
+    r.rows = (int)min64(BM, cnt - first);
     return r;
 }
 
@@ -310,19 +371,21 @@ __device__ __noinline__ void fused_weight_sum(const Params& p, bool valid, int64
     }
 }
 
-template <int WQ>
-__global__ void __launch_bounds__(Fmt<WQ>::THREADS, 1)
+template <int WQ, int CG>
+__global__ void __launch_bounds__(Cfg<WQ, CG>::THREADS, 1)
 tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b0,
                const __grid_constant__ CUtensorMap tm_b1, const __grid_constant__ CUtensorMap tm_out, const Params p) {
     pdl_enter();
-    using L = Layout<WQ>;
+    using C = Cfg<WQ, CG>;
+    using L = Layout<WQ, CG>;
     constexpr int STAGES = L::STAGES;
-    constexpr int RAW = Fmt<WQ>::RAW_BYTES;
+    constexpr int RAW = C::RAW;
+    constexpr int BH = C::B_HELD;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
     uint8_t* sA = smem;
     uint8_t* sB = smem + STAGES * A_BYTES;
-    uint8_t* sR = smem + STAGES * (A_BYTES + B_BYTES);  // raw quantised B tiles
+    uint8_t* sR = smem + STAGES * (A_BYTES + BH);  // raw quantised B tiles
     uint8_t* sE = smem + STAGES * L::STAGE_BYTES;  // output staging (L::EPI_BYTES)
     uint64_t* bars = reinterpret_cast<uint64_t*>(sE + L::EPI_BYTES);
     uint64_t* full = bars;                 // TMA landed (A + B or A + raw B)
@@ -335,65 +398,79 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t rank = CG == 2 ? cluster_rank() : 0u;  // 0: this CTA issues the MMAs
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(&full[s], 1);
             mbar_init(&empty[s], 1);
-            mbar_init(&conv[s], CONVERT_WARPS);
+            mbar_init(&conv[s], C::CONVERT_WARPS ? C::CONVERT_WARPS : 1);
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(&tfull[a], 1);
-            mbar_init(&tempty[a], 4 * 32);
+            mbar_init(&tempty[a], 4 * CG);  // one arrival per epilogue warp of each CTA
         }
         mbar_init(drain, 1);
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
-    if (warp == 1) {
-        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
-                     "r"(TMEM_COLS)
-                     : "memory");
-        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
-    }
+    if (warp == 1) tmem_alloc<CG>(tmem_slot);
     tc_fence_before();
     __syncthreads();
+    if constexpr (CG == 2) cluster_sync();  // both CTAs' barriers exist before either signals the other
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
 
     const int total = p.sched[1] * p.n_tiles;
     const int nkb = p.K / BK;
+    const int unit = blockIdx.x / CG, n_units = gridDim.x / CG;  // CTA pairs walk the list together
 
     if (warp == 0 && lane == 0) {
         // ---------------------------------------------------- TMA producer
+        // CG = 2: both CTAs' copies of a slot complete on the even CTA's
+        // full barrier, which expects the bytes of both
         int stage = 0;
         uint32_t phase = 0;
         uint32_t inflight = 0, inflight_par = 0;  // stages loaded but not seen consumed
         bool ok = true;
-        for (int w = blockIdx.x; w < total && ok; w += gridDim.x) {
-            const Work wk = decode_work(p, w);
+        for (int w = unit; w < total && ok; w += n_units) {
+            const Work wk = decode_work<CG>(p, w, rank);
             int b0, b1;
             b_rows(p, wk, b0, b1);
+            // CG = 2: this CTA's half of the B tile (gate rows / up rows, or down rows 0-127 / 128-255)
+            const CUtensorMap* tm_bh = rank ? &tm_b1 : &tm_b0;
+            const int bh = rank ? b1 : b0;
             for (int kb = 0; kb < nkb; ++kb) {
                 if (WQ == GBMOE_FP8_E4M3_B128 && kb + kFp8PrefetchAhead < nkb) {
                     // fp8 tiles wait on the decode as well as on the load: bring the
                     // k-block a few stages ahead into L2 so its TMA load returns sooner
                     const int xp = (kb + kFp8PrefetchAhead) * BK;
                     tma_prefetch_2d(&tm_a, xp, (int)wk.row0);
-                    tma_prefetch_2d(&tm_b0, xp, b0);
-                    tma_prefetch_2d(&tm_b1, xp, b1);
+                    if (CG == 1) {
+                        tma_prefetch_2d(&tm_b0, xp, b0);
+                        tma_prefetch_2d(&tm_b1, xp, b1);
+                    } else {
+                        tma_prefetch_2d(tm_bh, xp, bh);
+                    }
                 }
                 if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, p.err, p.wait_limit_ns)) { ok = false; break; }
                 inflight &= ~(1u << stage);
-                mbar_expect_tx(&full[stage], A_BYTES + (RAW ? RAW : B_BYTES));
-                tma_load_2d(sA + stage * A_BYTES, &tm_a, kb * BK, (int)wk.row0, &full[stage]);
-                if (RAW == 0) {
-                    tma_load_2d(sB + stage * B_BYTES, &tm_b0, kb * BK, b0, &full[stage]);
-                    tma_load_2d(sB + stage * B_BYTES + B_BYTES / 2, &tm_b1, kb * BK, b1, &full[stage]);
+                if (rank == 0) mbar_expect_tx(&full[stage], CG * (A_BYTES + (RAW ? RAW : BH)));
+                if (rank == 0) tma_load_2d(sA + stage * A_BYTES, &tm_a, kb * BK, (int)wk.row0, &full[stage]);
+                else tma_load_2d_to_pair_leader(sA + stage * A_BYTES, &tm_a, kb * BK, (int)wk.row0, &full[stage]);
+                // raw boxes are BK elements wide: BK bytes (fp8) or BK/2 bytes (int4, MXFP4)
+                const int xr = packed4<WQ>() ? kb * (BK / 2) : kb * BK;
+                if (CG == 1) {
+                    if (RAW == 0) {
+                        tma_load_2d(sB + stage * BH, &tm_b0, kb * BK, b0, &full[stage]);
+                        tma_load_2d(sB + stage * BH + BH / 2, &tm_b1, kb * BK, b1, &full[stage]);
+                    } else {
+                        tma_load_2d(sR + stage * RAW, &tm_b0, xr, b0, &full[stage]);
+                        tma_load_2d(sR + stage * RAW + RAW / 2, &tm_b1, xr, b1, &full[stage]);
+                    }
+                } else if (rank == 0) {
+                    tma_load_2d(sB + stage * BH, tm_bh, kb * BK, bh, &full[stage]);
                 } else {
-                    // raw boxes are BK elements wide: BK bytes (fp8) or BK/2 bytes (int4)
-                    const int x = packed4<WQ>() ? kb * (BK / 2) : kb * BK;
-                    tma_load_2d(sR + stage * RAW, &tm_b0, x, b0, &full[stage]);
-                    tma_load_2d(sR + stage * RAW + RAW / 2, &tm_b1, x, b1, &full[stage]);
+                    tma_load_2d_to_pair_leader(sB + stage * BH, tm_bh, kb * BK, bh, &full[stage]);
                 }
                 inflight |= 1u << stage;
                 inflight_par = (inflight_par & ~(1u << stage)) | (phase << stage);
@@ -402,10 +479,17 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
         }
         // let every copy issued land before the CTA leaves: after a normal run
         // these phases have completed already; after an abort (here or in
-        // another role) the last loads may still be in flight
-        for (int s = 0; s < STAGES; ++s)
-            if ((inflight >> s) & 1u) drain_wait(&full[s], (inflight_par >> s) & 1u);
-    } else if (warp == 1 && lane == 0) {
+        // another role) the last loads may still be in flight. The odd CTA of
+        // a pair sees its copies only through the even CTA's barrier: it waits
+        // for the release of those slots instead (the MMAs that read them
+        // finished), which also keeps the even CTA's last arrivals on this
+        // CTA's barriers before it leaves.
+        for (int s = 0; s < STAGES; ++s) {
+            if (!((inflight >> s) & 1u)) continue;
+            if (rank == 0) drain_wait(&full[s], (inflight_par >> s) & 1u);
+            if (CG == 2) drain_wait(&empty[s], (inflight_par >> s) & 1u);
+        }
+    } else if (warp == 1 && lane == 0 && rank == 0) {
         // ------------------------------------------------------ MMA issuer
         int stage = 0;
         uint32_t phase = 0;
@@ -413,8 +497,12 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
         uint32_t acc_phase = 0;
         bool ok = true;
         bool issued = false;
-        for (int w = blockIdx.x; w < total && ok; w += gridDim.x) {
-            if (!mbar_wait(&tempty[acc], acc_phase ^ 1, abort_flag, p.err, p.wait_limit_ns)) { ok = false; break; }
+        for (int w = unit; w < total && ok; w += n_units) {
+            if (!(CG == 1 ? mbar_wait(&tempty[acc], acc_phase ^ 1, abort_flag, p.err, p.wait_limit_ns)
+                          : mbar_wait_cluster(&tempty[acc], acc_phase ^ 1, abort_flag, p.err, p.wait_limit_ns))) {
+                ok = false;
+                break;
+            }
             tc_fence_after();
             const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
             for (int kb = 0; kb < nkb; ++kb) {
@@ -422,23 +510,23 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
                 if (RAW && !mbar_wait(&conv[stage], phase, abort_flag, p.err, p.wait_limit_ns)) { ok = false; break; }
                 tc_fence_after();
                 const uint64_t da = sw128_desc(smem_u32(sA + stage * A_BYTES));
-                const uint64_t db = sw128_desc(smem_u32(sB + stage * B_BYTES));
+                const uint64_t db = sw128_desc(smem_u32(sB + stage * BH));
 #pragma unroll
                 for (int j = 0; j < BK / 16; ++j)  // +32 bytes along K per slice
-                    mma_bf16(d_tmem, da + 2 * j, db + 2 * j, (kb | j) != 0 ? 1u : 0u);
+                    mma_bf16<CG>(d_tmem, da + 2 * j, db + 2 * j, (kb | j) != 0 ? 1u : 0u);
                 issued = true;
-                mma_commit(&empty[stage]);
+                commit_to<CG>(&empty[stage], 0x3);
                 if (++stage == STAGES) { stage = 0; phase ^= 1; }
             }
             if (!ok) break;
-            mma_commit(&tfull[acc]);
+            commit_to<CG>(&tfull[acc], 0x3);
             if (++acc == 2) { acc = 0; acc_phase ^= 1; }
         }
         if (issued) {
             // every MMA issued has finished before TMEM is released (after a
             // normal run the epilogue has seen them all; after an abort in
             // another role this issuer may have run up to two tiles ahead)
-            mma_commit(drain);
+            commit_to<CG>(drain, 0x1);
             drain_wait(drain, 0);
         }
     } else if (warp >= 2 && warp < 6) {
@@ -449,8 +537,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
         int sbuf = 0;
         int acc = 0;
         uint32_t acc_phase = 0;
-        for (int w = blockIdx.x; w < total; w += gridDim.x) {
-            const Work wk = decode_work(p, w);
+        for (int w = unit; w < total; w += n_units) {
+            const Work wk = decode_work<CG>(p, w, rank);
             if (!warp_wait(&tfull[acc], acc_phase, abort_flag, p.err, p.wait_limit_ns)) break;
             tc_fence_after();
             const uint32_t t_row = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
@@ -504,23 +592,29 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
                     store_bf16x32(dst + c, v);
                 }
             }
+            // this warp's reads of the accumulator are done: one arrival on the
+            // issuing CTA's barrier (for a pair, possibly the other CTA's)
             tc_fence_before();
-            mbar_arrive(&tempty[acc]);
+            __syncwarp();
+            if (lane == 0) {
+                if (CG == 1) mbar_arrive(&tempty[acc]);
+                else mbar_arrive_rank(&tempty[acc], 0);
+            }
             if (p.fuse_k) fused_weight_sum(p, valid, pair, col0);  // warp-uniform
             if (++acc == 2) { acc = 0; acc_phase ^= 1; }
         }
         if (lane == 0) bulk_wait_all();  // stores complete before the CTA exits
     } else if (RAW && warp >= 6) {
         // ------------------------------------------- weight decode (B rows)
-        const int r = threadIdx.x - 6 * 32;  // B row 0..255 of the tile
-        const int half = r >> 7;
+        const int r = threadIdx.x - 6 * 32;  // B row 0 .. C::B_ROWS-1 held by this CTA
+        const int half = CG == 2 ? (int)rank : r >> 7;
         const void* scales = half ? p.scale1 : p.scale0;
         const int kgroups = p.K / 128;
         int stage = 0;
         uint32_t phase = 0;
         bool ok = true;
-        for (int w = blockIdx.x; w < total && ok; w += gridDim.x) {
-            const Work wk = decode_work(p, w);
+        for (int w = unit; w < total && ok; w += n_units) {
+            const Work wk = decode_work<CG>(p, w, rank);
             int b0, b1;
             b_rows(p, wk, b0, b1);
             const int64_t brow = (half ? b1 : b0) + (r & 127);  // absolute row of the stacked B tensor
@@ -545,7 +639,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
                 }
                 if (!warp_wait(&full[stage], phase, abort_flag, p.err, p.wait_limit_ns)) { ok = false; break; }
                 const uint8_t* raw = sR + stage * RAW;
-                uint8_t* dstB = sB + stage * B_BYTES;
+                uint8_t* dstB = sB + stage * BH;
                 if (WQ == GBMOE_FP8_E4M3_B128) {
 #pragma unroll
                     for (int c = 0; c < 4; ++c) {
@@ -587,10 +681,12 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
     }
     tc_fence_before();
     __syncthreads();
+    // a pair: neither CTA releases TMEM or leaves while the other may still
+    // signal its barriers or the MMAs may still write its TMEM
+    if constexpr (CG == 2) cluster_sync();
     if (warp == 1) {
         tc_fence_after();
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(TMEM_COLS)
-                     : "memory");
+        tmem_dealloc<CG>(tmem_base);
     }
 }
 
@@ -696,32 +792,65 @@ static bool map_weights(CUtensorMap* m, int wq, const void* base, int64_t rows, 
     }
 }
 
+template <int WQ, int CG>
+static cudaError_t set_smem_attr() {
+    static DeviceOnce smem_set;
+    return smem_set.run([] {
+        return cudaFuncSetAttribute(tc_gemm_kernel<WQ, CG>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    Layout<WQ, CG>::SMEM_BYTES);
+    });
+}
+
+// CTA pairs of the CG = 2 kernel for WQ that fit on the device at once
+// (queried once per device), 0 when none does
 template <int WQ>
+static int pair_units() {
+    static std::atomic<int> cache[kMaxDevices];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return 0;
+    if (const int n = cache[dev].load(std::memory_order_relaxed); n > 0) return n;
+    if (set_smem_attr<WQ, 2>() != cudaSuccess) return 0;
+    const int n = max_active_clusters(tc_gemm_kernel<WQ, 2>, Cfg<WQ, 2>::THREADS, Layout<WQ, 2>::SMEM_BYTES, 2);
+    if (n > 0) cache[dev].store(n, std::memory_order_relaxed);
+    return n;
+}
+
+template <int WQ, int CG>
 static cudaError_t launch_gemm_t(const CUtensorMap& a, const CUtensorMap& b0, const CUtensorMap& b1,
                                  const CUtensorMap& out, const Params& prm, int64_t max_work, cudaStream_t stream) {
-    static DeviceOnce smem_set;
-    cudaError_t e = smem_set.run([] {
-        return cudaFuncSetAttribute(tc_gemm_kernel<WQ>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    Layout<WQ>::SMEM_BYTES);
-    });
-    if (e != cudaSuccess) return e;
-    const int grid = (int)min64(sm_count(), max_work);
+    if (const cudaError_t e = set_smem_attr<WQ, CG>(); e != cudaSuccess) return e;
+    int units;  // persistent CTAs, or CTA pairs
+    if constexpr (CG == 1) units = sm_count();
+    else units = pair_units<WQ>();
+    if (units <= 0) return cudaErrorNotSupported;
+    const int grid = (int)min64(units, max_work) * CG;
     if (grid <= 0) return cudaSuccess;
-    if (const cudaError_t le = launch_k(tc_gemm_kernel<WQ>, dim3(grid), dim3(Fmt<WQ>::THREADS),
-            Layout<WQ>::SMEM_BYTES, stream, a, b0, b1, out, prm); le != cudaSuccess)
-        return le;
+    cudaError_t le;
+    if (CG == 1)
+        le = launch_k(tc_gemm_kernel<WQ, CG>, dim3(grid), dim3(Cfg<WQ, CG>::THREADS), Layout<WQ, CG>::SMEM_BYTES,
+                      stream, a, b0, b1, out, prm);
+    else
+        le = launch_k_cluster(tc_gemm_kernel<WQ, CG>, dim3(grid), dim3(Cfg<WQ, CG>::THREADS),
+                              Layout<WQ, CG>::SMEM_BYTES, stream, 2, a, b0, b1, out, prm);
+    if (le != cudaSuccess) return le;
     return cudaGetLastError();
 }
 
+template <int CG>
 static cudaError_t launch_gemm(int wq, const CUtensorMap& a, const CUtensorMap& b0, const CUtensorMap& b1,
                                const CUtensorMap& out, const Params& prm, int64_t max_work, cudaStream_t stream) {
-    switch (wq) {
-        case GBMOE_BF16: return launch_gemm_t<GBMOE_BF16>(a, b0, b1, out, prm, max_work, stream);
-        case GBMOE_FP8_E4M3_B128:
-            return launch_gemm_t<GBMOE_FP8_E4M3_B128>(a, b0, b1, out, prm, max_work, stream);
-        case GBMOE_INT4_G128: return launch_gemm_t<GBMOE_INT4_G128>(a, b0, b1, out, prm, max_work, stream);
-        case GBMOE_MXFP4: return launch_gemm_t<GBMOE_MXFP4>(a, b0, b1, out, prm, max_work, stream);
-        default: return cudaErrorInvalidValue;
+    if constexpr (CG == 2) {
+        if (wq != GBMOE_BF16) return cudaErrorNotSupported;
+        return launch_gemm_t<GBMOE_BF16, 2>(a, b0, b1, out, prm, max_work, stream);
+    } else {
+        switch (wq) {
+            case GBMOE_BF16: return launch_gemm_t<GBMOE_BF16, 1>(a, b0, b1, out, prm, max_work, stream);
+            case GBMOE_FP8_E4M3_B128:
+                return launch_gemm_t<GBMOE_FP8_E4M3_B128, 1>(a, b0, b1, out, prm, max_work, stream);
+            case GBMOE_INT4_G128: return launch_gemm_t<GBMOE_INT4_G128, 1>(a, b0, b1, out, prm, max_work, stream);
+            case GBMOE_MXFP4: return launch_gemm_t<GBMOE_MXFP4, 1>(a, b0, b1, out, prm, max_work, stream);
+            default: return cudaErrorInvalidValue;
+        }
     }
 }
 
@@ -731,6 +860,14 @@ bool ffn_tc_supported(const FfnProblem& p) {
     const bool wq_ok = p.w_dtype == GBMOE_BF16 || p.w_dtype == GBMOE_FP8_E4M3_B128 ||
                        p.w_dtype == GBMOE_INT4_G128 || p.w_dtype == GBMOE_MXFP4;
     return p.act_dtype == GBMOE_BF16 && wq_ok && p.H % 256 == 0 && p.I % 128 == 0 && tc::encode_fn() != nullptr;
+}
+
+// the CTA-pair kernel runs this problem on the current device: its B tiles
+// are bf16 (bf16 weights, or a decode-once copy: w_dq set)
+bool ffn_tc_pair_supported(const FfnProblem& p) {
+    if (!ffn_tc_supported(p)) return false;
+    if (p.w_dtype != GBMOE_BF16 && !p.w_dq) return false;
+    return tc::pair_units<GBMOE_BF16>() > 0;
 }
 
 // Decodes gate, up and down of the active experts into the bf16 copy w_dq
@@ -778,13 +915,14 @@ cudaError_t launch_gate_tc(const void* x, const void* wg, const float* bias, flo
     g.out = nullptr; g.err = err; g.scale0 = g.scale1 = nullptr;
     g.wait_limit_ns = tc_wait_limit_ns();
     g.out_f32 = logits; g.col_bias = bias; g.f32_cols = E;
-    return launch_gemm(GBMOE_BF16, ma, mb, mb, mo, g, sched_max_tiles(1, T, BM) * g.n_tiles, stream);
+    return launch_gemm<1>(GBMOE_BF16, ma, mb, mb, mo, g, sched_max_tiles(1, T, BM) * g.n_tiles, stream);
 }
 
 cudaError_t launch_ffn_tc(const FfnProblem& pin, cudaStream_t stream) {
     using namespace tc;
     if (pin.n_rows == 0) return cudaSuccess;
-    cudaError_t err = launch_ffn_schedule(pin.counts, pin.E, pin.n_rows, BM, pin.sched, stream);
+    const int tile_m = pin.cta_pair ? 2 * BM : BM;  // M tile of one CTA, or of a CTA pair
+    cudaError_t err = launch_ffn_schedule(pin.counts, pin.E, pin.n_rows, tile_m, pin.sched, stream);
     if (err != cudaSuccess) return err;
     FfnProblem p = pin;
     if (pin.w_dq && (pin.w_dtype == GBMOE_FP8_E4M3_B128 || pin.w_dtype == GBMOE_INT4_G128 ||
@@ -805,7 +943,7 @@ cudaError_t launch_ffn_tc(const FfnProblem& pin, cudaStream_t stream) {
         a_rows = p.x_sorted;
     }
 
-    const int64_t max_m = sched_max_tiles(p.E, p.n_rows, BM);
+    const int64_t max_m = sched_max_tiles(p.E, p.n_rows, tile_m);
     CUtensorMap ma, mg, mu, mh, md, oh, oy;
     if (!map_bf16(&ma, a_rows, p.n_rows, p.H) || !map_weights(&mg, p.w_dtype, p.w_gate, (int64_t)p.E * p.I, p.H) ||
         !map_weights(&mu, p.w_dtype, p.w_up, (int64_t)p.E * p.I, p.H) || !map_bf16(&mh, p.h, p.n_rows, p.I) ||
@@ -819,7 +957,8 @@ cudaError_t launch_ffn_tc(const FfnProblem& pin, cudaStream_t stream) {
     g.out = static_cast<__nv_bfloat16*>(p.h); g.err = p.err;
     g.scale0 = p.s_gate; g.scale1 = p.s_up;
     g.wait_limit_ns = tc_wait_limit_ns();
-    if ((err = launch_gemm(p.w_dtype, ma, mg, mu, oh, g, max_m * g.n_tiles, stream)) != cudaSuccess) return err;
+    auto gemm = pin.cta_pair ? launch_gemm<2> : launch_gemm<1>;
+    if ((err = gemm(p.w_dtype, ma, mg, mu, oh, g, max_m * g.n_tiles, stream)) != cudaSuccess) return err;
 
     Params d = g;
     d.K = p.I; d.n_tiles = p.H / BN; d.out_cols = p.H; d.b_rows_per_expert = p.H; d.swiglu = 0;
@@ -833,7 +972,7 @@ cudaError_t launch_ffn_tc(const FfnProblem& pin, cudaStream_t stream) {
         d.out_final = static_cast<__nv_bfloat16*>(p.out_final);
         d.arrive = p.arrive;
     }
-    return launch_gemm(p.w_dtype, mh, md, md, oy, d, max_m * d.n_tiles, stream);
+    return gemm(p.w_dtype, mh, md, md, oy, d, max_m * d.n_tiles, stream);
 }
 
 }  // namespace gbmoe

@@ -62,6 +62,7 @@ struct FfnProblem {
     float* a_s;                 //   and their 1x128 scales [n_rows, H/128]
     void* h_q;                  //   h the same way, [2, n_rows, I]
     float* h_s;                 //   and its 1x128 scales [n_rows, I/128]
+    int cta_pair;               // tensor-core routes: 1 = CTA pairs (cta_group::2, 256-row M tiles)
     int32_t* sched;             // schedule ints, ffn_sched_ints(E, n_rows)
     int32_t* err;               // device error word
     // Weight Sum fused into the down GEMM (tensor-core routes; fuse_k = top_k,
@@ -77,6 +78,7 @@ struct FfnProblem {
 
 size_t ffn_sched_ints(int E, int64_t n_rows);
 constexpr int64_t kDequantRowsPerExpert = 256;  // AUTO: TC_DEQUANT from this many rows per expert
+constexpr int64_t kPairRowsPerExpert = 1024;    // AUTO: CTA pairs from this many rows per expert
 cudaError_t launch_ffn_stream(const FfnProblem& p, cudaStream_t stream);
 size_t stream_smem_bytes(int act_dtype, int H, int I);  // per CTA, streaming route
 // dynamic shared memory a CTA may use on sm_103a (227 KB); a streaming problem
@@ -85,6 +87,7 @@ constexpr size_t stream_smem_budget() { return 227 * 1024; }
 cudaError_t launch_ffn_simt(const FfnProblem& p, cudaStream_t stream);
 cudaError_t launch_ffn_tc(const FfnProblem& p, cudaStream_t stream);
 bool ffn_tc_supported(const FfnProblem& p);
+bool ffn_tc_pair_supported(const FfnProblem& p);
 cudaError_t launch_ffn_tc_fp8(const FfnProblem& p, cudaStream_t stream);
 bool ffn_tc_fp8_supported(const FfnProblem& p);
 

@@ -71,7 +71,9 @@ def test_workload_configs_are_valid(lib, wid):
     (dict(ffn_route=gb.FFN_TC), gb.EUNSUPPORTED),  # fp32 activations have no tensor-core route
     (dict(ffn_route=gb.FFN_TC_DEQUANT), gb.EUNSUPPORTED),
     (dict(ffn_route=gb.FFN_TC_FP8), gb.EUNSUPPORTED),  # fp8 route needs fp8 weights and bf16 activations
-    (dict(ffn_route=6), gb.EINVAL),
+    (dict(ffn_route=gb.FFN_TC_PAIR), gb.EUNSUPPORTED),
+    (dict(ffn_route=gb.FFN_TC_PAIR_DEQUANT), gb.EUNSUPPORTED),
+    (dict(ffn_route=8), gb.EINVAL),
     (dict(gate_route=3), gb.EINVAL),
     (dict(gate_route=gb.GATE_TC), gb.EUNSUPPORTED),  # the tensor-core gate takes bf16 activations
     (dict(combine_route=3), gb.EINVAL),

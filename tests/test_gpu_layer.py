@@ -18,9 +18,10 @@ from gpu_helpers import (act_np, assert_close, config, rel_err, tiles_covered, t
 
 pytestmark = pytest.mark.gpu
 
-ROUTES = {1: ["simt", "stream", "auto"], 2: ["stream", "simt", "auto"], 3: ["simt", "auto"],
-          4: ["simt", "auto", "tc", "tc_dequant"], 5: ["simt", "auto", "tc"], 6: ["simt", "auto", "tc_dequant"]}
-ALL_ROUTES = ["auto", "stream", "simt", "tc", "tc_dequant", "tc_fp8"]
+ROUTES = {1: ["simt", "stream", "auto"], 2: ["stream", "simt", "auto"], 3: ["simt", "auto", "tc", "tc_pair"],
+          4: ["simt", "auto", "tc", "tc_dequant"], 5: ["simt", "auto", "tc", "tc_pair_dequant"],
+          6: ["simt", "auto", "tc_dequant", "tc_pair_dequant"]}
+ALL_ROUTES = ["auto", "stream", "simt", "tc", "tc_dequant", "tc_fp8", "tc_pair", "tc_pair_dequant"]
 
 
 @pytest.fixture(scope="module", params=[1, 2, 3, 4, 5, 6])
@@ -116,7 +117,7 @@ def test_forward_matches_oracle(wcase, route):
     assert np.array_equal(ids.cpu().numpy(), ref["topk_ids"])
     assert np.array_equal(counts.cpu().numpy(), ref["counts"])
     assert len(ref["rows"]) == wl.T  # every token compared
-    if gb.ffn_route(config(wl, route)) in ("tc", "tc_dequant", "tc_fp8"):
+    if gb.ffn_route(config(wl, route)) in ("tc", "tc_dequant", "tc_fp8", "tc_pair", "tc_pair_dequant"):
         cov, total = tiles_covered(ref["topk_ids"], ref["rows"], ref["counts"], ref["sorted_pair"], ref["offsets"])
         assert cov == total, f"compared tokens reach {cov} of {total} (expert, M tile) pairs"
     assert_close(act_np(out), ref["out"], tol_for(wl), f"workload {wid} route {route}")

@@ -31,16 +31,39 @@ def forward(wl, dev, route):
     return out, ids
 
 
+def pair_route(wq):
+    """The CTA-pair route of a weight format: pairs multiply bf16 B tiles, so
+    quantised weights take the decode-once pair route."""
+    return "tc_pair" if wq == "bf16" else "tc_pair_dequant"
+
+
+@pytest.mark.parametrize("pair", [False, True])
 @pytest.mark.parametrize("wq", ["bf16", "fp8_b128", "int4_g128", "mxfp4"])
 @pytest.mark.parametrize("T,E,k,H,I", [(200, 4, 2, 512, 256), (1000, 4, 2, 256, 384), (333, 16, 3, 768, 128)])
-def test_tc_small_ragged(T, E, k, H, I, wq):
+def test_tc_small_ragged(T, E, k, H, I, wq, pair):
     wl = BASE.replace(T=T, E=E, top_k=k, H=H, I=I, seed=T + E, wq=wq)
     inp = synth.make_inputs(wl)
     dev = to_device(wl, inp)
-    out, ids = forward(wl, dev, "tc")
+    out, ids = forward(wl, dev, pair_route(wq) if pair else "tc")
     ref = oracle.forward(wl, inp)
     assert np.array_equal(ids.cpu().numpy(), ref["topk_ids"])
     assert_close(act_np(out), ref["out"], tol_for(wl))
+
+
+@pytest.mark.parametrize("wq", ["bf16", "int4_g128"])
+@pytest.mark.parametrize("T,E,k,H,I", [(1000, 4, 2, 256, 384), (333, 16, 3, 768, 128), (77, 3, 3, 512, 256)])
+def test_pair_route_equals_single_cta_route(T, E, k, H, I, wq):
+    """A CTA pair's 256-row MMA sums each output element over the same k
+    slices in the same order as the one-CTA 128-row MMA, and the decoded
+    operands are the same, so the two routes give bit-identical outputs
+    (expert tails of 1..255 rows, including pairs whose odd CTA has none)."""
+    wl = BASE.replace(T=T, E=E, top_k=k, H=H, I=I, seed=T + 3 * E, wq=wq)
+    inp = synth.make_inputs(wl)
+    dev = to_device(wl, inp)
+    out1, ids1 = forward(wl, dev, "tc" if wq == "bf16" else "tc_dequant")
+    out2, ids2 = forward(wl, dev, pair_route(wq))
+    assert torch.equal(ids1, ids2)
+    assert torch.equal(out1.view(torch.int16), out2.view(torch.int16))
 
 
 def test_tc_sigmoid_grouped_fp8_with_shared_expert():
@@ -66,6 +89,8 @@ def test_dequant_route_equals_in_gemm_decode(T, E, k, H, I, wq):
     out_dq, ids_dq = forward(wl, dev, "tc_dequant")
     assert torch.equal(ids_tc, ids_dq)
     assert torch.equal(out_tc.view(torch.int16), out_dq.view(torch.int16))
+    out_pq, _ = forward(wl, dev, "tc_pair_dequant")  # the same on CTA pairs
+    assert torch.equal(out_tc.view(torch.int16), out_pq.view(torch.int16))
     ref = oracle.forward(wl, inp)
     assert_close(act_np(out_dq), ref["out"], tol_for(wl))
 
@@ -86,18 +111,19 @@ def test_dequant_route_with_shared_expert_and_inactive_experts():
 def test_auto_route_choice():
     """AUTO: streaming for decode; fp8 weights on the fp8 tensor-core route;
     int4/MXFP4 decoded in the GEMM for few rows per expert, decoded once for
-    many."""
+    many; CTA pairs for deep experts (>= 1024 rows each)."""
     assert gb.ffn_route(config(synth.WORKLOADS[2])) == "stream"
     assert gb.ffn_route(config(synth.WORKLOADS[3])) == "tc"
     assert gb.ffn_route(config(synth.WORKLOADS[4])) == "tc_fp8"
     assert gb.ffn_route(config(synth.WORKLOADS[4]), shared=True) == "tc_fp8"
-    assert gb.ffn_route(config(synth.WORKLOADS[5])) == "tc_dequant"
+    assert gb.ffn_route(config(synth.WORKLOADS[5])) == "tc_pair_dequant"  # 1536 rows per expert: CTA pairs
     assert gb.ffn_route(config(synth.WORKLOADS[6])) == "tc"
-    assert gb.ffn_route(config(synth.WORKLOADS[6]), shared=True) == "tc_dequant"
+    assert gb.ffn_route(config(synth.WORKLOADS[6]), shared=True) == "tc_pair_dequant"
 
 
+@pytest.mark.parametrize("pair", [False, True])
 @pytest.mark.parametrize("wq", ["bf16", "int4_g128"])
-def test_bounded_wait_timeout_is_reported_and_the_next_call_is_clean(wq, monkeypatch):
+def test_bounded_wait_timeout_is_reported_and_the_next_call_is_clean(wq, pair, monkeypatch):
     """With the tensor-core kernels' wait limit lowered to 0 ns, a wait that
     is not over at once gives up (the first accumulator alone takes tens of
     microseconds): the kernel stops, drains what it issued, frees its TMEM and
@@ -107,7 +133,7 @@ def test_bounded_wait_timeout_is_reported_and_the_next_call_is_clean(wq, monkeyp
     wl = BASE.replace(T=333, E=16, top_k=3, H=768, I=128, seed=401, wq=wq)
     inp = synth.make_inputs(wl)
     dev = to_device(wl, inp)
-    cfg = config(wl, "tc")
+    cfg = config(wl, pair_route(wq) if pair else "tc")
     ws = workspace(cfg)
     out = torch.empty((wl.T, wl.H), dtype=torch.bfloat16, device="cuda")
     args = (cfg, dev["x"], dev["w_router"], dev["logit_bias"], dev["select_bias"], wbundle(dev["experts"]), None,
