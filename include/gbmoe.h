@@ -170,6 +170,12 @@ typedef struct gbmoe_expert_weights {
 /* Human-readable name of a status code (static string). */
 const char* gbmoe_status_string(int status);
 
+/* The CUDA runtime error code (a cudaError_t value) behind the last
+ * GBMOE_ECUDA this thread received from the library, or 0 if none; the
+ * library links its own copy of the CUDA runtime, so the caller's
+ * cudaGetLastError does not see it. Cleared by reading. */
+int gbmoe_last_cuda_error(void);
+
 /* GBMOE_OK if the config is valid and covered, else the status a call with it
  * would return. Limits: H % 256 == 0, I % 128 == 0 (I_shared too),
  * 1 <= E <= 512, 1 <= top_k <= min(E, 32), T >= 0, P <= 2^30. */

@@ -34,13 +34,17 @@ EXPORTS = ("gbmoe_status_string", "gbmoe_check_config", "gbmoe_workspace_size", 
            "gbmoe_gate_route", "moe_route",
            "moe_permute",
            "moe_grouped_ffn", "moe_shared_ffn", "moe_combine", "moe_forward", "moe_forward_hostio",
-           "moe_device_status", "moe_permute_noalloc")
+           "moe_device_status", "moe_permute_noalloc", "gbmoe_last_cuda_error")
 
 
 class GbmoeError(RuntimeError):
     def __init__(self, status: int, call: str):
         self.status = status
-        super().__init__(f"{call}: {status_string(status)} ({status})")
+        detail = ""
+        if status == ECUDA:  # the CUDA error code behind it
+            self.cuda_error = lib().gbmoe_last_cuda_error()
+            detail = f", cudaError {self.cuda_error}"
+        super().__init__(f"{call}: {status_string(status)} ({status}{detail})")
 
 
 class Config(ctypes.Structure):
@@ -72,6 +76,8 @@ def lib() -> ctypes.CDLL:
         sz = ctypes.c_size_t
         L.gbmoe_status_string.argtypes = [ctypes.c_int]
         L.gbmoe_status_string.restype = ctypes.c_char_p
+        L.gbmoe_last_cuda_error.argtypes = []
+        L.gbmoe_last_cuda_error.restype = ctypes.c_int
         L.gbmoe_check_config.argtypes = [cfgp]
         L.gbmoe_workspace_size.argtypes = [cfgp]
         L.gbmoe_workspace_size.restype = sz

@@ -153,7 +153,13 @@ T* at(void* ws, size_t off) {
     return reinterpret_cast<T*>(static_cast<char*>(ws) + off);
 }
 
-int cuda_status(cudaError_t e) { return e == cudaSuccess ? GBMOE_OK : GBMOE_ECUDA; }
+thread_local int g_last_cuda_error = 0;  // gbmoe_last_cuda_error
+
+int cuda_status(cudaError_t e) {
+    if (e == cudaSuccess) return GBMOE_OK;
+    g_last_cuda_error = (int)e;
+    return GBMOE_ECUDA;
+}
 
 int check_ws(const gbmoe_config* c, void* ws, size_t bytes) {
     if (!ws || !aligned(ws, kAlign)) return GBMOE_EINVAL;
@@ -290,6 +296,12 @@ FfnProblem shared_problem(const gbmoe_config* c, const void* x, const gbmoe_expe
 
 extern "C" {
 
+int gbmoe_last_cuda_error(void) {
+    const int e = g_last_cuda_error;
+    g_last_cuda_error = 0;
+    return e;
+}
+
 const char* gbmoe_status_string(int s) {
     switch (s) {
         case GBMOE_OK: return "ok";
@@ -417,7 +429,7 @@ int moe_forward(const gbmoe_config* cfg, const void* x, const void* w_router, co
     if ((s = route_launchable(cfg, r_routed, cfg->I))) return s;
     const int r_shared = cfg->has_shared ? pick_route(cfg, cfg->T, 1, cfg->I_shared) : GBMOE_FFN_SIMT;
     if (cfg->has_shared && (s = route_launchable(cfg, r_shared, cfg->I_shared))) return s;
-    if (cudaMemsetAsync(at<int32_t>(ws, L.err), 0, 4, st) != cudaSuccess) return GBMOE_ECUDA;
+    if (const cudaError_t ce = cudaMemsetAsync(at<int32_t>(ws, L.err), 0, 4, st); ce != cudaSuccess) return cuda_status(ce);
     int32_t* ids = at<int32_t>(ws, L.ids);
     float* w = at<float>(ws, L.w);
     int32_t* counts = at<int32_t>(ws, L.counts);
@@ -441,8 +453,8 @@ int moe_forward(const gbmoe_config* cfg, const void* x, const void* w_router, co
     const bool fused = cfg->combine_route == GBMOE_COMBINE_FUSED &&
                        bf16_gemm_route(r_routed);
     if (fused) {  // Weight Sum in the down GEMM's epilogue
-        if (cudaMemsetAsync(at<int32_t>(ws, L.arrive), 0, (size_t)cfg->T * (cfg->H / 256) * 4, st) != cudaSuccess)
-            return GBMOE_ECUDA;
+        if ((s = cuda_status(cudaMemsetAsync(at<int32_t>(ws, L.arrive), 0, (size_t)cfg->T * (cfg->H / 256) * 4, st))))
+            return s;
         pr.fuse_k = cfg->top_k;
         pr.topk_w = w;
         pr.y_shared = ysh;
@@ -453,12 +465,11 @@ int moe_forward(const gbmoe_config* cfg, const void* x, const void* w_router, co
     if (!fused &&
         (s = cuda_status(launch_combine(y, w, pos, ysh, out, cfg->T, cfg->top_k, cfg->H, cfg->act_dtype, st))))
         return s;
-    if (topk_ids && cudaMemcpyAsync(topk_ids, ids, P * 4, cudaMemcpyDeviceToDevice, st) != cudaSuccess)
-        return GBMOE_ECUDA;
-    if (topk_w && cudaMemcpyAsync(topk_w, w, P * 4, cudaMemcpyDeviceToDevice, st) != cudaSuccess) return GBMOE_ECUDA;
-    if (counts_out && cudaMemcpyAsync(counts_out, counts, (size_t)cfg->E * 4, cudaMemcpyDeviceToDevice, st) !=
-                          cudaSuccess)
-        return GBMOE_ECUDA;
+    if (topk_ids && (s = cuda_status(cudaMemcpyAsync(topk_ids, ids, P * 4, cudaMemcpyDeviceToDevice, st)))) return s;
+    if (topk_w && (s = cuda_status(cudaMemcpyAsync(topk_w, w, P * 4, cudaMemcpyDeviceToDevice, st)))) return s;
+    if (counts_out &&
+        (s = cuda_status(cudaMemcpyAsync(counts_out, counts, (size_t)cfg->E * 4, cudaMemcpyDeviceToDevice, st))))
+        return s;
     return GBMOE_OK;
 }
 
@@ -475,12 +486,11 @@ int moe_forward_hostio(const gbmoe_config* cfg, const void* x_host, const void* 
     const size_t bytes = (size_t)cfg->T * cfg->H * act_bytes(cfg->act_dtype);
     void* xin = at<char>(ws, L.xin);
     void* xout = at<char>(ws, L.xout);
-    if (bytes && cudaMemcpyAsync(xin, x_host, bytes, cudaMemcpyHostToDevice, st) != cudaSuccess) return GBMOE_ECUDA;
+    if (bytes && (s = cuda_status(cudaMemcpyAsync(xin, x_host, bytes, cudaMemcpyHostToDevice, st)))) return s;
     s = moe_forward(cfg, xin, w_router, logit_bias, select_bias, experts, shared, xout, nullptr, nullptr, nullptr, ws,
                     ws_bytes, stream);
     if (s) return s;
-    if (bytes && cudaMemcpyAsync(out_host, xout, bytes, cudaMemcpyDeviceToHost, st) != cudaSuccess)
-        return GBMOE_ECUDA;
+    if (bytes && (s = cuda_status(cudaMemcpyAsync(out_host, xout, bytes, cudaMemcpyDeviceToHost, st)))) return s;
     return GBMOE_OK;
 }
 
@@ -488,9 +498,9 @@ int moe_device_status(void* ws, void* stream, int32_t* status) {
     if (!ws || !status || !aligned(ws, kAlign)) return GBMOE_EINVAL;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     int32_t word = 0;
-    if (cudaStreamSynchronize(st) != cudaSuccess) return GBMOE_ECUDA;
-    if (cudaMemcpy(&word, ws, 4, cudaMemcpyDeviceToHost) != cudaSuccess) return GBMOE_ECUDA;
-    if (cudaMemset(ws, 0, 4) != cudaSuccess) return GBMOE_ECUDA;
+    if (const cudaError_t ce = cudaStreamSynchronize(st); ce != cudaSuccess) return cuda_status(ce);
+    if (const cudaError_t ce = cudaMemcpy(&word, ws, 4, cudaMemcpyDeviceToHost); ce != cudaSuccess) return cuda_status(ce);
+    if (const cudaError_t ce = cudaMemset(ws, 0, 4); ce != cudaSuccess) return cuda_status(ce);
     *status = word ? GBMOE_EDEVICE_TIMEOUT : GBMOE_OK;
     return GBMOE_OK;
 }

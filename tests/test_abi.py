@@ -168,3 +168,11 @@ def test_forced_stream_route_checks_the_shared_expert_before_launching(lib):
     assert e.value.status == gb.EUNSUPPORTED
     c.I_shared = 2048  # fits: the same call passes the checks (it would launch, so it is not made here)
     assert gb.check_config(c) == gb.OK
+
+
+def test_last_cuda_error_starts_clear(lib):
+    """No CUDA call has failed in this thread: the recorded code is 0, and a
+    call that fails on its arguments (not in CUDA) leaves it 0."""
+    assert gb.lib().gbmoe_last_cuda_error() == 0
+    assert gb.check_config(cfg_of(1, T=-1)) == gb.EINVAL
+    assert gb.lib().gbmoe_last_cuda_error() == 0
