@@ -345,13 +345,14 @@ tc_fp8_gemm_kernel(const __grid_constant__ CUtensorMap tm_a1, const __grid_const
                 if (!warp_wait(&pfull[pb], pph, abort_flag, p.err, p.wait_limit_ns)) { ok = false; break; }
                 tc_fence_after();
                 const uint32_t tb = t_row + pb * BN;
+                // 16 columns at a time: next to 128 accumulators, wider loads spill
 #pragma unroll
-                for (int part = 0; part < 4; ++part) {
-                    float v[32];
-                    tmem_ld32(tb + (uint32_t)((part < 2 ? c0 : c1) + 32 * (part & 1)), v);
-                    const float f = part < 2 ? f0 : f1;
+                for (int part = 0; part < 8; ++part) {
+                    float v[16];
+                    tmem_ld16(tb + (uint32_t)((part < 4 ? c0 : c1) + 16 * (part & 3)), v);
+                    const float f = part < 4 ? f0 : f1;
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) acc[32 * part + i] = fmaf(v[i], f, acc[32 * part + i]);
+                    for (int i = 0; i < 16; ++i) acc[16 * part + i] = fmaf(v[i], f, acc[16 * part + i]);
                 }
                 tc_fence_before();
                 __syncwarp();
