@@ -49,14 +49,12 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # (python bench.py --workload W --set ... --profile 1 under
 # ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum,gpu__time_duration.sum):
 #   decode   T=8 E=32 (29 active):    stream gate/up + down            1.0966 GB
-#   prefill  T=2048 E=32 (32 active): gather + gate/up GEMM + down GEMM  1.7653 GB
 #   fp8      T=512 E=64 (64 active):  quantise, gate/up, quantise, down  3.0185 GB
 #   MXFP4    T=512 E=64 (64 active):  gather + gate/up GEMM + down GEMM  1.6565 GB
 # (the skewed int4 workload's offsets exist for its full size only, so its
 # reduced case differs in I and is not scaled here)
 TRAFFIC_PER_ACTIVE_EXPERT: dict = {
     ("decode_bf16_T32_H4096_E128_k8_I1536", "stream"): 1.0966e9 / 29,
-    ("prefill_bf16_T8192_H4096_E128_k8_I1536", "tc"): 1.7653e9 / 32,
     ("dsv3_fp8_T2048_H7168_E256s1_k8_I2048", "tc_fp8"): 3.0185e9 / 64,
     ("dsv4_mxfp4_T2048_H7168_E256s1_k8_I2048", "tc"): 1.6565e9 / 64,
 }
@@ -261,13 +259,15 @@ def launches_per_step(wl, route: str, shared_route) -> int:
     """Kernels this library launches per layer forward: gate logits + expert
     choice, the permutation (one kernel up to 1024 pairs, else three), per FFN
     problem a schedule kernel + 2 GEMM/stream kernels (+ a row gather for the
-    routed experts on the tensor-core routes, + 3 weight-decode passes on the
-    decode-once route), and the combine."""
+    routed experts on the CTA-pair routes, whose GEMM does not gather its rows
+    itself, + 3 weight-decode passes on the decode-once routes), and the
+    combine."""
     def ffn(r, routed):
         if r == "tc_fp8":  # schedule, x quantisation, gate/up GEMM, h quantisation, down GEMM
             return 5
-        gemm = r in ("tc", "tc_dequant", "tc_pair", "tc_pair_dequant")
-        return 3 + (1 if routed and gemm else 0) + (3 if r in ("tc_dequant", "tc_pair_dequant") else 0)
+        # the one-CTA bf16 GEMM gathers its own rows; decoding GEMMs and pairs use the gather kernel
+        gather = r in ("tc_pair", "tc_pair_dequant") or (r == "tc" and wl.wq != "bf16")
+        return 3 + (1 if routed and gather else 0) + (3 if r in ("tc_dequant", "tc_pair_dequant") else 0)
 
     n = 2 + (1 if wl.P <= 1024 else 3) + ffn(route, True) + 1
     if shared_route is not None:
@@ -400,9 +400,9 @@ def measure(args, wid: int, overrides, dist, world: int, rank: int, local: int, 
     routed_bytes = algorithmic_weight_bytes(wl.replace(has_shared=False), active)
     flops = 6.0 * wl.P * wl.H * wl.I
     kernel = {"stream": "moe_grouped_ffn, weight-streaming route (gate/up + down)",
-              "tc": "moe_grouped_ffn, tcgen05 route (row gather + gate/up GEMM with SwiGLU + down GEMM)",
-              "tc_dequant": "moe_grouped_ffn, tcgen05 decode-once route (3 weight-decode passes + row gather + "
-                            "gate/up GEMM with SwiGLU + down GEMM)",
+              "tc": "moe_grouped_ffn, tcgen05 route (gate/up GEMM gathering its rows, with SwiGLU + down GEMM)",
+              "tc_dequant": "moe_grouped_ffn, tcgen05 decode-once route (3 weight-decode passes + gate/up GEMM "
+                            "gathering its rows, with SwiGLU + down GEMM)",
               "tc_fp8": "moe_grouped_ffn, fp8 tcgen05 route (two-term e4m3 quantisation of the rows + gate/up "
                         "GEMM with per-k-block promotion and SwiGLU + quantisation of h + down GEMM)",
               "tc_pair": "moe_grouped_ffn, tcgen05 CTA-pair route (row gather + gate/up GEMM with SwiGLU + down "

@@ -88,7 +88,12 @@ struct Cfg {
     static constexpr int B_HELD = B_BYTES / CG;          // bf16 B bytes per stage of one CTA
     static constexpr int B_ROWS = BN / CG;               // B rows of one CTA
     static constexpr int CONVERT_WARPS = RAW ? B_ROWS / 32 : 0;  // one thread per B row
-    static constexpr int THREADS = 192 + CONVERT_WARPS * 32;
+    // bf16, one CTA: four warps can gather the A rows from x themselves (one
+    // thread per row; 10 warps keep a thread's 168 registers)
+    static constexpr bool GATHER = WQ == GBMOE_BF16 && CG == 1;
+    static constexpr int GATHER_WARPS = GATHER ? BM / 32 : 0;
+    static constexpr int GATHER_AHEAD = 2;  // k blocks a gather warp keeps in flight before signalling
+    static constexpr int THREADS = 192 + CONVERT_WARPS * 32 + GATHER_WARPS * 32;
     static constexpr int STAGES = CG == 1 ? (WQ == GBMOE_FP8_E4M3_B128 ? 3 : 4) : (RAW ? 5 : 6);
 };
 
@@ -138,7 +143,18 @@ struct Params {
     const __nv_bfloat16* y_shared;
     __nv_bfloat16* out_final;
     int32_t* arrive;
+    // A rows gathered from x by the kernel (Cfg::GATHER; null: A by TMA):
+    // row r of the sorted order is x row a_gather[r] / a_gather_div (a
+    // negative entry, and rows past n_rows, read x row 0; never stored)
+    const int32_t* a_gather;
+    int a_gather_div;
+    const __nv_bfloat16* a_src;  // x [*, K]
 };
+
+// 16-byte global -> shared copy through L2 (cp.async), tracked by commit groups
+__device__ __forceinline__ void cp_async_16(void* dst, const void* src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
 
 // Instruction descriptor, kind::f16: fp32 accumulator (bits 4-5 = 1), bf16 A
 // and B (bits 7-9, 10-12 = 1), both K-major, N/8 in bits 17-22, M/16 in 24-28
@@ -400,8 +416,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t rank = CG == 2 ? cluster_rank() : 0u;  // 0: this CTA issues the MMAs
     if (threadIdx.x == 0) {
+        const bool gathering = C::GATHER && p.a_gather != nullptr;
         for (int s = 0; s < STAGES; ++s) {
-            mbar_init(&full[s], 1);
+            mbar_init(&full[s], gathering ? 1 + C::GATHER_WARPS : 1);  // + one arrival per gather warp
             mbar_init(&empty[s], 1);
             mbar_init(&conv[s], C::CONVERT_WARPS ? C::CONVERT_WARPS : 1);
         }
@@ -454,9 +471,14 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
                 }
                 if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, p.err, p.wait_limit_ns)) { ok = false; break; }
                 inflight &= ~(1u << stage);
-                if (rank == 0) mbar_expect_tx(&full[stage], CG * (A_BYTES + (RAW ? RAW : BH)));
-                if (rank == 0) tma_load_2d(sA + stage * A_BYTES, &tm_a, kb * BK, (int)wk.row0, &full[stage]);
-                else tma_load_2d_to_pair_leader(sA + stage * A_BYTES, &tm_a, kb * BK, (int)wk.row0, &full[stage]);
+                const bool gather_a = C::GATHER && p.a_gather != nullptr;  // the gather warps bring A
+                if (rank == 0) mbar_expect_tx(&full[stage], CG * ((gather_a ? 0 : A_BYTES) + (RAW ? RAW : BH)));
+                if (gather_a) {
+                } else if (rank == 0) {
+                    tma_load_2d(sA + stage * A_BYTES, &tm_a, kb * BK, (int)wk.row0, &full[stage]);
+                } else {
+                    tma_load_2d_to_pair_leader(sA + stage * A_BYTES, &tm_a, kb * BK, (int)wk.row0, &full[stage]);
+                }
                 // raw boxes are BK elements wide: BK bytes (fp8) or BK/2 bytes (int4, MXFP4)
                 const int xr = packed4<WQ>() ? kb * (BK / 2) : kb * BK;
                 if (CG == 1) {
@@ -678,6 +700,57 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
                 if (++stage == STAGES) { stage = 0; phase ^= 1; }
             }
         }
+    }
+    if (C::GATHER && warp >= 6 + C::CONVERT_WARPS && p.a_gather != nullptr) {
+        // ----------------------------------------------- A row gather
+        // warp g copies A rows 32g .. 32g+31 of each k block (64 bf16 = 128
+        // bytes a row) from their x rows into the 128-byte-swizzled slot, four
+        // whole rows per instruction (lane l: row 4i + l/8, 16-byte chunk l%8);
+        // a warp signals a slot once its copies of it landed (GATHER_AHEAD k
+        // blocks later), after a proxy fence that makes them visible to the MMAs
+        constexpr int D = C::GATHER_AHEAD;
+        static_assert(D < STAGES, "a gather warp must signal a slot before it needs that slot again");
+        const int row_base = (warp - 6 - C::CONVERT_WARPS) * 32 + (lane >> 3);
+        const int chunk = lane & 7;
+        int stage = 0;
+        uint32_t phase = 0;
+        int64_t issued = 0;
+        bool ok = true;
+        for (int w = unit; w < total && ok; w += n_units) {
+            const Work wk = decode_work<CG>(p, w, rank);
+            const __nv_bfloat16* src[8];  // this lane's chunk of rows row_base + 4i
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const int64_t prow = wk.row0 + row_base + 4 * i;
+                int32_t tok = 0;
+                if (prow < p.n_rows) {
+                    const int32_t sp = p.a_gather[prow];
+                    tok = sp >= 0 ? sp / p.a_gather_div : 0;
+                }
+                src[i] = p.a_src + (int64_t)tok * p.K + 8 * chunk;
+            }
+            for (int kb = 0; kb < nkb; ++kb) {
+                if (!warp_wait(&empty[stage], phase ^ 1, abort_flag, p.err, p.wait_limit_ns)) { ok = false; break; }
+                uint8_t* dst = sA + stage * A_BYTES;
+#pragma unroll
+                for (int i = 0; i < 8; ++i) cp_async_16(dst + sw128_off(row_base + 4 * i, chunk), src[i] + kb * BK);
+                asm volatile("cp.async.commit_group;" ::: "memory");
+                if (++issued > D) {  // the k block D back has landed: signal its slot
+                    asm volatile("cp.async.wait_group %0;" ::"n"(D) : "memory");
+                    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&full[(stage + STAGES - D) % STAGES]);
+                }
+                if (++stage == STAGES) { stage = 0; phase ^= 1; }
+            }
+        }
+        // the last k blocks' copies land before the CTA leaves; after a normal
+        // run their slots are signalled too
+        asm volatile("cp.async.wait_group 0;" ::: "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        __syncwarp();
+        if (ok && lane == 0)
+            for (int64_t i = issued > D ? issued - D : 0; i < issued; ++i) mbar_arrive(&full[i % STAGES]);
     }
     tc_fence_before();
     __syncthreads();
@@ -928,10 +1001,12 @@ cudaError_t launch_ffn_tc(const FfnProblem& pin, cudaStream_t stream) {
     if (pin.w_dq && (pin.w_dtype == GBMOE_FP8_E4M3_B128 || pin.w_dtype == GBMOE_INT4_G128 ||
                      pin.w_dtype == GBMOE_MXFP4))
         if ((err = dequant_all(pin, p, stream)) != cudaSuccess) return err;
-    // A operand of the gate/up GEMM: x rows in sorted order (a gathered copy),
-    // or x itself when rows are already in order (no sorted_pair: shared expert)
+    // A operand of the gate/up GEMM: x rows in sorted order. The one-CTA bf16
+    // GEMM gathers them from x itself; otherwise a gathered copy (x itself
+    // when rows are already in order: no sorted_pair, the shared expert)
     const void* a_rows = p.x;
-    if (p.sorted_pair) {
+    const bool self_gather = p.sorted_pair && !pin.cta_pair && p.w_dtype == GBMOE_BF16;
+    if (p.sorted_pair && !self_gather) {
         const int vpr = p.H * 2 / 16;
         const int64_t nvec = p.n_rows * vpr;
         const int gblocks = (int)min64((nvec + 255) / 256, 152 * 16);
@@ -945,7 +1020,9 @@ cudaError_t launch_ffn_tc(const FfnProblem& pin, cudaStream_t stream) {
 
     const int64_t max_m = sched_max_tiles(p.E, p.n_rows, tile_m);
     CUtensorMap ma, mg, mu, mh, md, oh, oy;
-    if (!map_bf16(&ma, a_rows, p.n_rows, p.H) || !map_weights(&mg, p.w_dtype, p.w_gate, (int64_t)p.E * p.I, p.H) ||
+    // (with self_gather the A map is unused; it still spans only x's own rows)
+    const int64_t a_map_rows = self_gather ? p.n_rows / p.pair_div : p.n_rows;
+    if (!map_bf16(&ma, a_rows, a_map_rows, p.H) || !map_weights(&mg, p.w_dtype, p.w_gate, (int64_t)p.E * p.I, p.H) ||
         !map_weights(&mu, p.w_dtype, p.w_up, (int64_t)p.E * p.I, p.H) || !map_bf16(&mh, p.h, p.n_rows, p.I) ||
         !map_weights(&md, p.w_dtype, p.w_down, (int64_t)p.E * p.H, p.I) || !map_out(&oh, p.h, p.n_rows, p.I) ||
         !map_out(&oy, p.y, p.n_rows, p.H))
@@ -957,10 +1034,16 @@ cudaError_t launch_ffn_tc(const FfnProblem& pin, cudaStream_t stream) {
     g.out = static_cast<__nv_bfloat16*>(p.h); g.err = p.err;
     g.scale0 = p.s_gate; g.scale1 = p.s_up;
     g.wait_limit_ns = tc_wait_limit_ns();
+    if (self_gather) {
+        g.a_gather = p.sorted_pair;
+        g.a_gather_div = p.pair_div;
+        g.a_src = static_cast<const __nv_bfloat16*>(p.x);
+    }
     auto gemm = pin.cta_pair ? launch_gemm<2> : launch_gemm<1>;
     if ((err = gemm(p.w_dtype, ma, mg, mu, oh, g, max_m * g.n_tiles, stream)) != cudaSuccess) return err;
 
     Params d = g;
+    d.a_gather = nullptr;  // the down GEMM reads h, already in sorted order
     d.K = p.I; d.n_tiles = p.H / BN; d.out_cols = p.H; d.b_rows_per_expert = p.H; d.swiglu = 0;
     d.out = static_cast<__nv_bfloat16*>(p.y);
     d.scale0 = p.s_down; d.scale1 = p.s_down;
