@@ -49,12 +49,14 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # (python bench.py --workload W --set ... --profile 1 under
 # ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum,gpu__time_duration.sum):
 #   decode   T=8 E=32 (29 active):    stream gate/up + down            1.0966 GB
+#   prefill  T=2048 E=32 (32 active): gate/up GEMM (own row gather) + down GEMM  1.6655 GB
 #   fp8      T=512 E=64 (64 active):  quantise, gate/up, quantise, down  3.0185 GB
 #   MXFP4    T=512 E=64 (64 active):  gather + gate/up GEMM + down GEMM  1.6565 GB
 # (the skewed int4 workload's offsets exist for its full size only, so its
 # reduced case differs in I and is not scaled here)
 TRAFFIC_PER_ACTIVE_EXPERT: dict = {
     ("decode_bf16_T32_H4096_E128_k8_I1536", "stream"): 1.0966e9 / 29,
+    ("prefill_bf16_T8192_H4096_E128_k8_I1536", "tc"): 1.6655e9 / 32,
     ("dsv3_fp8_T2048_H7168_E256s1_k8_I2048", "tc_fp8"): 3.0185e9 / 64,
     ("dsv4_mxfp4_T2048_H7168_E256s1_k8_I2048", "tc"): 1.6565e9 / 64,
 }

@@ -709,7 +709,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__
         // a warp signals a slot once its copies of it landed (GATHER_AHEAD k
         // blocks later), after a proxy fence that makes them visible to the MMAs
         constexpr int D = C::GATHER_AHEAD;
-        static_assert(D < STAGES, "a gather warp must signal a slot before it needs that slot again");
+        static_assert(!C::GATHER || D < STAGES, "a gather warp must signal a slot before it needs that slot again");
         const int row_base = (warp - 6 - C::CONVERT_WARPS) * 32 + (lane >> 3);
         const int chunk = lane & 7;
         int stage = 0;
