@@ -54,6 +54,8 @@ def _L():
         lib.oracle_get_threads.restype = ctypes.c_int
         lib.oracle_gate_logits.argtypes = [i64, i64, i64, vp, vp, vp, vp]
         lib.oracle_gate_logits.restype = ctypes.c_int
+        lib.oracle_rmsnorm.argtypes = [i64, i64, vp, vp, ctypes.c_float, vp]
+        lib.oracle_rmsnorm.restype = ctypes.c_int
         lib.oracle_pexp.argtypes = [ctypes.c_float]
         lib.oracle_pexp.restype = ctypes.c_float
         lib.oracle_pexp_n.argtypes = [i64, vp, vp]
@@ -111,6 +113,28 @@ def gate_logits(x: np.ndarray, w_router: np.ndarray, logit_bias=None) -> np.ndar
     if _L().oracle_gate_logits(T, H, E, _p(x), _p(g), _p(b), _p(out)) != 0:
         raise ValueError("gate logits need H % 256 == 0")
     return out
+
+
+def rmsnorm(x: np.ndarray, gamma: np.ndarray, eps: float) -> np.ndarray:
+    """fp32 RMSNorm of the rows of x [T, H] in the pinned order (see
+    oracle.c); the caller rounds the result to the activation dtype."""
+    x = _c(x, np.float32)
+    g = _c(gamma, np.float32)
+    T, H = x.shape
+    out = np.empty((T, H), dtype=np.float32)
+    if _L().oracle_rmsnorm(T, H, _p(x), _p(g), ctypes.c_float(eps), _p(out)) != 0:
+        raise ValueError("rmsnorm needs H % 256 == 0 and eps >= 0")
+    return out
+
+
+def round_bf16(v: np.ndarray) -> np.ndarray:
+    """Raw bf16 bit patterns (uint16) of fp32 values, rounded to nearest even
+    (a NaN stays a quiet NaN)."""
+    u = _c(v, np.float32).view(np.uint32).astype(np.uint64)
+    nan = (u & 0x7FFFFFFF) > 0x7F800000
+    r = ((u + 0x7FFF + ((u >> 16) & 1)) >> 16) & 0xFFFF
+    r = np.where(nan, ((u >> 16) | 0x40) & 0xFFFF, r)
+    return r.astype(np.uint16)
 
 
 def pexp(v: np.ndarray) -> np.ndarray:

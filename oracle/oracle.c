@@ -116,6 +116,46 @@ int oracle_gate_logits(int64_t T, int64_t H, int64_t E, const float* x, const fl
 }
 
 /*
+ * RMSNorm of the layer input before the gate (the step before the MoE Gate
+ * node): y = x / sqrt(mean(x^2) + eps) * gamma, the standard definition.
+ * Its result decides the expert choice (the logits are taken from it), so
+ * it is computed in fp32 in a fixed order the GPU reproduces (reading: the
+ * paper gives no formula): ss = sum of x^2 in the logits' order
+ * (pinned_dot(x, x)); ms = ss / H; v = ms + eps; r = sqrt(v); inv = 1 / r;
+ * y[h] = (x[h] * inv) * gamma[h]; every step one correctly rounded fp32
+ * operation. The caller rounds y to the activation dtype.
+ */
+typedef struct {
+    int64_t H;
+    const float *x, *gamma;
+    float eps;
+    float* y;
+} norm_ctx;
+
+static void norm_range(void* vp, int64_t b, int64_t e) {
+    norm_ctx* c = (norm_ctx*)vp;
+    for (int64_t t = b; t < e; ++t) {
+        const float* xr = c->x + t * c->H;
+        const float ss = pinned_dot(xr, xr, c->H);
+        const float ms = ss / (float)c->H;
+        const float v = ms + c->eps;
+        const float r = sqrtf(v);
+        const float inv = 1.0f / r;
+        for (int64_t h = 0; h < c->H; ++h) {
+            const float xs = xr[h] * inv;
+            c->y[t * c->H + h] = xs * c->gamma[h];
+        }
+    }
+}
+
+int oracle_rmsnorm(int64_t T, int64_t H, const float* x, const float* gamma, float eps, float* y) {
+    if (H % 256 != 0 || T < 0 || !(eps >= 0.0f)) return -1;
+    norm_ctx c = {H, x, gamma, eps, y};
+    parallel_for(T, norm_range, &c);
+    return 0;
+}
+
+/*
  * Pinned fp32 exponential, used where an exponential decides the expert
  * choice (sigmoid scores plus a selection bias). Written from the
  * mathematics, not from any library:
