@@ -195,6 +195,20 @@ int gbmoe_ffn_route(const gbmoe_config* cfg, int shared);
 int gbmoe_gate_route(const gbmoe_config* cfg);
 
 /*
+ * RMSNorm of the layer input, the step before the MoE Gate: for every row t,
+ *   y[t,:] = x[t,:] / sqrt(mean(x[t,:]^2) + eps) * gamma,
+ * in fp32 in the gate's fixed order (sum of squares: 32 partial sums over
+ * the 8-element chunks p, p+32, ... with one fused multiply-add per element,
+ * then the pairwise sums for d = 16..1; then mean, + eps, sqrt, reciprocal
+ * and the two products, each one correctly rounded fp32 operation), rounded
+ * once to act_dtype. Its output is the x that moe_route / moe_forward take:
+ * the experts' choice follows from it bit for bit. x, y [T, H] and gamma [H]
+ * are act_dtype device pointers (16-byte aligned; y may not overlap x);
+ * eps >= 0 and finite. Uses cfg's T, H and act_dtype only. No workspace.
+ */
+int moe_rmsnorm(const gbmoe_config* cfg, const void* x, const void* gamma, float eps, void* y, void* stream);
+
+/*
  * MoE Gate (Fig. 1 and Fig. 3). For every token t:
  *   l[t,e] = x[t,:] . w_router[e,:] (+ logit_bias[e]), fp32, in a fixed order:
  *     32 partial sums, partial p takes the 8-element chunks p, p+32, ... in

@@ -34,7 +34,7 @@ EXPORTS = ("gbmoe_status_string", "gbmoe_check_config", "gbmoe_workspace_size", 
            "gbmoe_gate_route", "moe_route",
            "moe_permute",
            "moe_grouped_ffn", "moe_shared_ffn", "moe_combine", "moe_forward", "moe_forward_hostio",
-           "moe_device_status", "moe_permute_noalloc", "gbmoe_last_cuda_error")
+           "moe_device_status", "moe_permute_noalloc", "gbmoe_last_cuda_error", "moe_rmsnorm")
 
 
 class GbmoeError(RuntimeError):
@@ -84,6 +84,7 @@ def lib() -> ctypes.CDLL:
         L.gbmoe_ffn_route.argtypes = [cfgp, ctypes.c_int]
         L.gbmoe_gate_route.argtypes = [cfgp]
         L.moe_route.argtypes = [cfgp, vp, vp, fp, fp, vp, vp, vp, sz, vp]
+        L.moe_rmsnorm.argtypes = [cfgp, vp, vp, ctypes.c_float, vp, vp]
         L.moe_permute.argtypes = [cfgp, vp, vp, vp, vp, vp, vp, sz, vp]
         L.moe_grouped_ffn.argtypes = [cfgp, vp, vp, vp, vp, wp, vp, vp, sz, vp]
         L.moe_shared_ffn.argtypes = [cfgp, vp, wp, vp, vp, sz, vp]
@@ -154,6 +155,11 @@ def ffn_route(cfg: Config, shared: bool = False) -> str:
     if r < 0:
         raise GbmoeError(r, "gbmoe_ffn_route")
     return {v: k for k, v in ROUTES.items()}[r]
+
+
+def moe_rmsnorm(cfg, x, gamma, eps, y, stream=None):
+    _check(lib().moe_rmsnorm(ctypes.byref(cfg), _ptr(x), _ptr(gamma), float(eps), _ptr(y), _stream(stream)),
+           "moe_rmsnorm")
 
 
 def moe_route(cfg, x, w_router, logit_bias, select_bias, topk_ids, topk_w, ws, stream=None):

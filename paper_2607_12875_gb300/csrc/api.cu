@@ -333,6 +333,19 @@ int gbmoe_gate_route(const gbmoe_config* cfg) {
     return s ? s : pick_gate(cfg);
 }
 
+int moe_rmsnorm(const gbmoe_config* cfg, const void* x, const void* gamma, float eps, void* y, void* stream) {
+    int s = check_cfg(cfg);
+    if (s) return s;
+    if (!(eps >= 0.0f) || !std::isfinite(eps)) return GBMOE_EINVAL;
+    if (cfg->T == 0) return GBMOE_OK;
+    if (!x || !gamma || !y || !aligned(x, 16) || !aligned(gamma, 16) || !aligned(y, 16)) return GBMOE_EINVAL;
+    const size_t bytes = (size_t)cfg->T * cfg->H * act_bytes(cfg->act_dtype);
+    const char *xb = static_cast<const char*>(x), *yb = static_cast<const char*>(y);
+    if (xb < yb + bytes && yb < xb + bytes) return GBMOE_EINVAL;  // overlapping rows
+    return cuda_status(launch_rmsnorm(x, gamma, eps, cfg->T, cfg->H, cfg->act_dtype, y,
+                                      static_cast<cudaStream_t>(stream)));
+}
+
 int moe_route(const gbmoe_config* cfg, const void* x, const void* w_router, const float* logit_bias,
               const float* select_bias, int32_t* topk_ids, float* topk_w, void* ws, size_t ws_bytes,
               void* stream) {

@@ -28,6 +28,9 @@ struct RouteScratch {
 cudaError_t launch_route(const RouteParams& rp, const void* x, const void* w_router, const float* logit_bias,
                          const float* select_bias, float* logits, int32_t* topk_ids, float* topk_w,
                          const RouteScratch& rs, cudaStream_t stream);
+// RMSNorm of x [T, H] (act dtype) with gamma [H] into y, in the gate's order
+cudaError_t launch_rmsnorm(const void* x, const void* gamma, float eps, int T, int H, int act_dtype, void* y,
+                           cudaStream_t stream);
 // router logits on the tensor cores (bf16 x and router weight; ffn_tc.cu)
 cudaError_t launch_gate_tc(const void* x, const void* wg, const float* bias, float* logits, int T, int H, int E,
                            int32_t* sched, int32_t* err, cudaStream_t stream);

@@ -465,6 +465,59 @@ static cudaError_t gate_tiled_smem() {
     });
 }
 
+// ------------------------------------------------ RMSNorm before the gate
+
+// y = x / sqrt(mean(x^2) + eps) * gamma per row, in the order of the gate's
+// logits (its output decides the routing): one warp per row; lane l takes
+// the 8-element chunks l, l+32, ... and sums their squares with one fused
+// multiply-add each; the 32 partial sums are combined by the butterfly of
+// pairwise additions; then ms = ss / H, v = ms + eps, r = sqrt(v), inv = 1 / r
+// and y = (x * inv) * gamma, every step one correctly rounded fp32
+// operation; y is rounded once to the activation type.
+template <typename TA>
+__global__ void __launch_bounds__(256)
+rmsnorm_kernel(const TA* __restrict__ x, const TA* __restrict__ gamma, float eps, int T, int H, TA* __restrict__ y) {
+    pdl_enter();
+    const int lane = threadIdx.x & 31;
+    const int64_t t = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
+    if (t >= T) return;
+    const TA* xr = x + t * H;
+    float ss = 0.0f;
+    for (int c = lane; c < H / 8; c += 32) {
+        float v[8];
+        Vec8<TA>::load(xr + 8 * c, v);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) ss = __fmaf_rn(v[i], v[i], ss);
+    }
+#pragma unroll
+    for (int d = 16; d >= 1; d >>= 1) ss = __fadd_rn(ss, __shfl_xor_sync(0xffffffffu, ss, d));
+    const float ms = __fdiv_rn(ss, (float)H);
+    const float inv = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(ms, eps)));
+    for (int c = lane; c < H / 8; c += 32) {
+        float v[8], g[8], o[8];
+        Vec8<TA>::load(xr + 8 * c, v);
+        Vec8<TA>::load(gamma + 8 * c, g);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) o[i] = __fmul_rn(__fmul_rn(v[i], inv), g[i]);
+        Vec8<TA>::store(y + t * H + 8 * c, o);
+    }
+}
+
+cudaError_t launch_rmsnorm(const void* x, const void* gamma, float eps, int T, int H, int act_dtype, void* y,
+                           cudaStream_t stream) {
+    if (T == 0) return cudaSuccess;
+    const dim3 grid((unsigned)((T + 7) / 8));
+    cudaError_t le;
+    if (act_dtype == GBMOE_BF16)
+        le = launch_k(rmsnorm_kernel<__nv_bfloat16>, grid, dim3(256), 0, stream, static_cast<const __nv_bfloat16*>(x),
+                      static_cast<const __nv_bfloat16*>(gamma), eps, T, H, static_cast<__nv_bfloat16*>(y));
+    else
+        le = launch_k(rmsnorm_kernel<float>, grid, dim3(256), 0, stream, static_cast<const float*>(x),
+                      static_cast<const float*>(gamma), eps, T, H, static_cast<float*>(y));
+    if (le != cudaSuccess) return le;
+    return cudaGetLastError();
+}
+
 cudaError_t launch_route(const RouteParams& rp, const void* x, const void* wg, const float* logit_bias,
                          const float* select_bias, float* logits, int32_t* topk_ids, float* topk_w,
                          const RouteScratch& rs, cudaStream_t stream) {

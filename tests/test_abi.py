@@ -176,3 +176,24 @@ def test_last_cuda_error_starts_clear(lib):
     assert gb.lib().gbmoe_last_cuda_error() == 0
     assert gb.check_config(cfg_of(1, T=-1)) == gb.EINVAL
     assert gb.lib().gbmoe_last_cuda_error() == 0
+
+
+def test_rmsnorm_rejects_bad_arguments_before_launching(lib):
+    """Null, misaligned or overlapping buffers and a negative or non-finite
+    eps are refused on the host (nothing reaches the GPU here)."""
+    c = cfg_of(1)  # T=64, H=256, fp32 activations: rows of 1 KB
+    x, g, y = FakePtr(), FakePtr(), FakePtr()
+    for args in [(None, g, 1e-6, y), (x, None, 1e-6, y), (x, g, 1e-6, None), (x, g, -1.0, y),
+                 (x, g, float("nan"), y), (x, g, float("inf"), y), (x, g, 1e-6, x)]:
+        with pytest.raises(gb.GbmoeError) as e:
+            gb.moe_rmsnorm(c, *args, stream=0)
+        assert e.value.status == gb.EINVAL
+
+    class Shifted(FakePtr):  # 8 bytes past an aligned address
+        def data_ptr(self):
+            return self.addr + 8
+    with pytest.raises(gb.GbmoeError) as e:
+        gb.moe_rmsnorm(c, Shifted(), g, 1e-6, y, stream=0)
+    assert e.value.status == gb.EINVAL
+    # T = 0: nothing to do, no pointer is needed
+    assert lib.moe_rmsnorm(ctypes.byref(cfg_of(1, T=0)), None, None, ctypes.c_float(1e-6), None, None) == gb.OK
