@@ -1,33 +1,36 @@
 // Fused MoE on tensor cores: grouped GEMMs with tcgen05, TMEM and TMA.
 //
-// Rows of each expert are contiguous after the permutation (the gate/up
-// GEMM reads a gathered copy of x in sorted order, the down GEMM reads h),
-// so every M tile is a plain 128-row box of a 2-D tensor. A tile that runs
-// past its expert's last row reads the next expert's rows (or TMA's zero
-// fill past the end); those rows are computed and never stored.
+// Rows of each expert are contiguous after the permutation, so every M tile
+// is a block of consecutive sorted rows of one expert. A tile that runs past
+// its expert's last row computes rows of the next expert (or zero fill past
+// the end); those rows are never stored.
 //
-// One persistent CTA per SM walks the (M tile, N tile) work list built on the
-// device. Warp roles (192 threads):
-//   warp 0    one lane issues TMA loads of A (128 x 64) and B (2 x 128 x 64)
-//             bf16 boxes, 128-byte swizzled, into a 4-stage shared ring;
+// One persistent CTA per SM (CG = 1) or per pair of SMs (CG = 2) walks the
+// (M tile, N tile) list built on the device. Warp roles:
+//   warp 0    one lane issues TMA loads into a ring of stages: the A tile
+//             (128 x 64 bf16, 128-byte swizzled) and the B tile (two 128-row
+//             halves: 128 gate + 128 up rows, or 256 down rows), or the raw
+//             quantised B tile instead of B;
 //   warp 1    allocates 512 TMEM columns (two 128 x 256 fp32 accumulators)
-//             and one lane issues tcgen05.mma (M=128, N=256, K=16) per
-//             16-wide slice, releasing ring slots and accumulators through
-//             tcgen05.commit -> mbarrier;
+//             and one lane issues tcgen05.mma (kind::f16, M=128 or 256 for a
+//             pair, N=256, K=16), releasing ring slots and accumulators
+//             through tcgen05.commit -> mbarrier;
 //   warps 2-5 read the accumulator with tcgen05.ld (warp w owns TMEM lanes
-//             32*(w%4)..+31, i.e. tile rows) and produce bf16 results:
-//             h = silu(gate) * up for the gate/up GEMM (B rows 0-127 are the
-//             gate rows, 128-255 the up rows of the same 128 columns), plain
-//             y for the down GEMM; each warp stages 32 rows x 32 columns in
-//             shared memory and writes them with one TMA store.
-// Quantised weights (fp8 e4m3 with 128x128 block scales, int4 with 128-wide
-// group scales, MXFP4 with 32-wide E8M0 scales) take the same path with eight
-// more warps: TMA brings the raw
-// weight tile (64- or 32-byte swizzled rows) next to the A tile, and
-// warps 6-13, one B row per thread, decode it, apply the scale and write
-// the bf16 operand in the 128-byte-swizzled layout the MMA reads, then
-// signal the MMA warp. This keeps quantised weights quantised in HBM. When
-// experts have many rows, so that several M tiles would decode the same
+//             32*(w%4)..+31, i.e. tile rows) and produce the results: h =
+//             silu(gate) * up for the gate/up GEMM, y for the down GEMM
+//             (TMA stores through a swizzled staging buffer), fp32 logits for
+//             the router, or the fused Weight Sum's weighted slots;
+//   warps 6+  quantised weights (fp8 e4m3 with 128x128 block scales, int4
+//             with 128-wide group scales, MXFP4 with 32-wide E8M0 scales):
+//             one thread per B row decodes the raw tile, applies the scale
+//             and writes the bf16 operand in the swizzled layout the MMA
+//             reads; bf16 weights on one CTA: four warps gather the A rows of
+//             the gate/up GEMM from x (cp.async), so no sorted copy of x is
+//             written.
+// A CTA pair (tcgen05 cta_group::2) shares each MMA: each CTA holds 128 A
+// rows and half of the B rows; the odd CTA's loads complete on the even
+// CTA's barriers and the even CTA's commits arrive on both CTAs' barriers.
+// When experts have many rows, so that several M tiles would decode the same
 // weight tile again, the caller's workspace instead receives one bf16 copy
 // of the active experts' weights (dequant_weights_kernel, same decode) and
 // the bf16 GEMM runs on it.

@@ -529,7 +529,8 @@ cudaError_t launch_route(const RouteParams& rp, const void* x, const void* wg, c
         // tensor-core logits, then the audited choice
         auto xp = static_cast<const __nv_bfloat16*>(x);
         auto wp = static_cast<const __nv_bfloat16*>(wg);
-        if (cudaMemsetAsync(rs.audit, 0, 8, stream) != cudaSuccess) return cudaErrorUnknown;  // norm max, count
+        if (const cudaError_t me = cudaMemsetAsync(rs.audit, 0, 8, stream); me != cudaSuccess)  // norm max, count
+            return me;
         if (const cudaError_t le = launch_k(row_norm_max_kernel, dim3((rp.E + 7) / 8), dim3(256), 0, stream, wp,
                 rp.E, rp.H, rs.audit); le != cudaSuccess)
             return le;
