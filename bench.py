@@ -412,6 +412,9 @@ def measure(args, wid: int, overrides, dist, world: int, rank: int, local: int, 
               "tc_pair_dequant": "moe_grouped_ffn, tcgen05 CTA-pair decode-once route (3 weight-decode passes + "
                                  "row gather + gate/up GEMM with SwiGLU + down GEMM, cta_group::2 MMAs)",
               "simt": "moe_grouped_ffn, CUDA-core route"}[route]
+    if route == "tc" and wl.wq != "bf16":  # decoding GEMMs read a gathered copy of x
+        kernel = ("moe_grouped_ffn, tcgen05 route (row gather + gate/up GEMM decoding its weight tiles, with "
+                  "SwiGLU + down GEMM)")
     tpe = TRAFFIC_PER_ACTIVE_EXPERT.get((wl.name, route))
     extra = {"traffic": None if tpe is None else tpe * active, "kernel": kernel, "active_experts": active,
              "route": route, "gate": gb.gate_route(cfg)}
