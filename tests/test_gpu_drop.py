@@ -57,7 +57,7 @@ def test_permute_drops_out_of_range_ids(T, k, E):
     assert (pp[~keep] == -1).all()
 
 
-@pytest.mark.parametrize("route", ["tc", "stream", "simt"])
+@pytest.mark.parametrize("route", ["tc", "tc_pair", "stream", "simt"])
 def test_ffn_and_combine_skip_dropped_pairs(route):
     wl = synth.WORKLOADS[1].replace(T=150, E=8, top_k=3, H=512, I=256, act="bf16", wq="bf16", seed=61)
     inp = synth.make_inputs(wl)

@@ -197,7 +197,7 @@ def test_fused_weight_sum_matches_oracle(wcase):
     within rounding of the separate combine."""
     wl, dev, ref = wcase["wl"], wcase["dev"], wcase["ref"]
     route = gb.ffn_route(config(wl))
-    if route not in ("tc", "tc_dequant"):
+    if route not in ("tc", "tc_dequant", "tc_pair", "tc_pair_dequant"):
         pytest.skip("the fused Weight Sum runs on the bf16 tensor-core routes")
     outs = []
     for comb in ("fused", "fused", "separate"):

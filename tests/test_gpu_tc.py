@@ -190,14 +190,16 @@ def test_tc_fp8_route_with_shared_expert_and_timeout():
 
 
 
+@pytest.mark.parametrize("pair", [False, True])
 @pytest.mark.parametrize("wq", ["bf16", "int4_g128"])
-def test_fused_weight_sum_small_with_shared_expert(wq):
+def test_fused_weight_sum_small_with_shared_expert(wq, pair):
     """Fused Weight Sum on a ragged problem with a shared expert (its row is
-    added by the warp that completes each token)."""
+    added by the warp that completes each token), on one-CTA and CTA-pair
+    GEMMs."""
     wl = BASE.replace(T=333, E=16, top_k=3, H=768, I=128, seed=211, wq=wq, has_shared=True, I_shared=256)
     inp = synth.make_inputs(wl)
     dev = to_device(wl, inp)
-    cfg = config(wl, "tc")
+    cfg = config(wl, pair_route(wq) if pair else "tc")
     cfg.combine_route = gb.COMBINE_FUSED
     ws = workspace(cfg)
     out = torch.empty((wl.T, wl.H), dtype=torch.bfloat16, device="cuda")
