@@ -99,6 +99,16 @@ size_t dequant_bytes(const gbmoe_config* c, int64_t n_rows, int E, int I) {
     return (size_t)3 * E * c->H * I * 2;
 }
 
+// Bytes of the sorted copy of x the routed problem's GEMM reads (0 when its
+// route does not read one: the one-CTA bf16 GEMM gathers its rows from x,
+// the other routes read x or the fp8 codes directly).
+size_t sorted_x_bytes(const gbmoe_config* c) {
+    const int64_t P = (int64_t)c->T * c->top_k;
+    const int r = pick_route(c, P, c->E, c->I);
+    const bool reads_copy = pair_route(r) || (r == GBMOE_FFN_TC && quantised_weights(c->w_dtype));
+    return reads_copy ? (size_t)P * c->H * act_bytes(c->act_dtype) : 0;
+}
+
 struct Layout {
     size_t err, audit, flagged, arrive, logits, ids, w, counts, offsets, sorted, pos, perm, sched, h, xs, y, ysh, xin, xout, wdq,
         wdq_sh, aq, as, hq, hs, total;
@@ -132,7 +142,7 @@ Layout layout(const gbmoe_config* c) {
     L.perm = take(permute_scratch_ints(P, (int)E) * 4);
     L.sched = take(ffn_sched_ints((int)(E > 1 ? E : 1), rows_max) * 4);
     L.h = take((size_t)rows_max * I_max * ab);
-    L.xs = take((size_t)rows_max * H * ab);
+    L.xs = take(sorted_x_bytes(c));
     L.y = take((size_t)P * H * ab);
     L.ysh = take(c->has_shared ? (size_t)T * H * ab : 0);
     L.xin = take((size_t)T * H * ab);
@@ -269,7 +279,8 @@ FfnProblem routed_problem(const gbmoe_config* c, const void* x, const int32_t* c
     p.w_gate = w->w_gate; p.w_up = w->w_up; p.w_down = w->w_down;
     p.s_gate = w->s_gate; p.s_up = w->s_up; p.s_down = w->s_down;
     p.y = y;
-    p.h = at<char>(ws, L.h); p.x_sorted = at<char>(ws, L.xs); p.sched = at<int32_t>(ws, L.sched);
+    p.h = at<char>(ws, L.h); p.sched = at<int32_t>(ws, L.sched);
+    p.x_sorted = sorted_x_bytes(c) ? at<char>(ws, L.xs) : nullptr;
     p.err = at<int32_t>(ws, L.err);
     p.w_dq = dequant_bytes(c, p.n_rows, p.E, p.I) ? at<char>(ws, L.wdq) : nullptr;
     set_fp8_buffers(p, L, ws);
@@ -285,7 +296,7 @@ FfnProblem shared_problem(const gbmoe_config* c, const void* x, const gbmoe_expe
     p.w_gate = w->w_gate; p.w_up = w->w_up; p.w_down = w->w_down;
     p.s_gate = w->s_gate; p.s_up = w->s_up; p.s_down = w->s_down;
     p.y = y;
-    p.h = at<char>(ws, L.h); p.x_sorted = at<char>(ws, L.xs); p.sched = at<int32_t>(ws, L.sched);
+    p.h = at<char>(ws, L.h); p.x_sorted = nullptr; p.sched = at<int32_t>(ws, L.sched);  // rows in order
     p.err = at<int32_t>(ws, L.err);
     p.w_dq = dequant_bytes(c, p.n_rows, p.E, p.I) ? at<char>(ws, L.wdq_sh) : nullptr;
     set_fp8_buffers(p, L, ws);

@@ -1010,6 +1010,7 @@ cudaError_t launch_ffn_tc(const FfnProblem& pin, cudaStream_t stream) {
     const void* a_rows = p.x;
     const bool self_gather = p.sorted_pair && !pin.cta_pair && p.w_dtype == GBMOE_BF16;
     if (p.sorted_pair && !self_gather) {
+        if (!p.x_sorted) return cudaErrorInvalidValue;  // the workspace holds no sorted copy for this route
         const int vpr = p.H * 2 / 16;
         const int64_t nvec = p.n_rows * vpr;
         const int gblocks = (int)min64((nvec + 255) / 256, 152 * 16);

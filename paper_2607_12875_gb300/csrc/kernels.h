@@ -57,7 +57,8 @@ struct FfnProblem {
     void* y;                    // [n_rows, H] act
     // scratch carved by the caller
     void* h;                    // [n_rows, I] act
-    void* x_sorted;             // [n_rows, H] act (tensor-core route only)
+    void* x_sorted;             // [n_rows, H] act: the sorted copy the quantised-weight one-CTA GEMM and the
+                                // CTA-pair GEMMs read (null on routes that do not use one)
     void* w_dq;                 // bf16 [E, I, H] gate, [E, I, H] up, [E, H, I] down, or null:
                                 // quantised weights are then decoded once into it (TC_DEQUANT)
     void* a_q;                  // fp8 route (TC_FP8): x rows in sorted order as two e4m3 code planes

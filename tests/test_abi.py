@@ -142,12 +142,15 @@ def test_entry_points_reject_bad_arguments_before_launching(lib):
 @pytest.mark.parametrize("wid", [4, 5, 6])
 def test_dequant_route_workspace_holds_bf16_weight_copies(lib, wid):
     """Forcing the decode-once route adds one bf16 copy of every expert's
-    gate, up and down matrices (and of the shared expert's) to the workspace."""
+    gate, up and down matrices (and of the shared expert's) to the workspace,
+    and drops the sorted copy of x that the in-GEMM decode route reads (the
+    bf16 GEMM after the decode pass gathers its rows itself)."""
     wl = synth.WORKLOADS[wid]
     tc = gb.workspace_size(cfg_of(wid, ffn_route=gb.FFN_TC))
     dq = gb.workspace_size(cfg_of(wid, ffn_route=gb.FFN_TC_DEQUANT))
     copies = 3 * wl.E * wl.H * wl.I * 2 + (3 * wl.H * wl.I_shared * 2 if wl.has_shared else 0)
-    assert copies <= dq - tc <= copies + 2 * 256
+    sorted_x = wl.P * wl.H * 2
+    assert copies - sorted_x <= dq - tc <= copies - sorted_x + 3 * 256
 
 
 def test_forced_stream_route_checks_the_shared_expert_before_launching(lib):
@@ -197,3 +200,19 @@ def test_rmsnorm_rejects_bad_arguments_before_launching(lib):
     assert e.value.status == gb.EINVAL
     # T = 0: nothing to do, no pointer is needed
     assert lib.moe_rmsnorm(ctypes.byref(cfg_of(1, T=0)), None, None, ctypes.c_float(1e-6), None, None) == gb.OK
+
+
+def test_sorted_copy_of_x_only_where_a_gemm_reads_it(lib):
+    """The one-CTA bf16 GEMM gathers its rows from x, so its workspace holds
+    no sorted copy of x; the CTA-pair GEMM and the one-CTA GEMM on quantised
+    weights read one (P x H activations)."""
+    wl = synth.WORKLOADS[3]
+    copy = wl.P * wl.H * 2
+    one = gb.workspace_size(cfg_of(3, ffn_route=gb.FFN_TC))
+    pair = gb.workspace_size(cfg_of(3, ffn_route=gb.FFN_TC_PAIR))
+    assert copy <= pair - one <= copy + 256
+    w5 = synth.WORKLOADS[5]
+    in_gemm = gb.workspace_size(cfg_of(5, ffn_route=gb.FFN_TC))             # decodes int4 in the GEMM
+    dq = gb.workspace_size(cfg_of(5, ffn_route=gb.FFN_TC_DEQUANT))         # bf16 copy, then gathers
+    weights_copy = 3 * w5.E * w5.H * w5.I * 2
+    assert dq - in_gemm == pytest.approx(weights_copy - w5.P * w5.H * 2, abs=512)
