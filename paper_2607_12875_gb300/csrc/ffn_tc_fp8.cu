@@ -22,8 +22,9 @@
 // One persistent CTA per SM walks the (M tile, N tile) list built on the
 // device. Warp roles (320 threads):
 //   warp 0    one lane issues TMA loads of q1 and q2 (128 rows x 128 e4m3
-//             each) and B (2 x 128 rows x 128 e4m3), 128-byte swizzled, into
-//             a 3-stage ring;
+//             each, as two 64-row boxes: the second only when the tile holds
+//             rows there) and B (2 x 128 rows x 128 e4m3), 128-byte
+//             swizzled, into a 3-stage ring;
 //   warp 1    allocates 512 TMEM columns (two 128 x 256 fp32 partial sums)
 //             and one lane issues tcgen05.mma (M=128, N=256, K=32): four for
 //             q1 and four for q2 per 128-wide k block, alternating between
@@ -247,12 +248,20 @@ tc_fp8_gemm_kernel(const __grid_constant__ CUtensorMap tm_a1, const __grid_const
             const Work wk = decode_work(p, w);
             int b0, b1;
             b_rows(p, wk, b0, b1);
+            // A in two 64-row boxes; the second only when the tile has rows
+            // there (the MMA's rows past the tile's end read whatever the slot
+            // held, and their accumulators are never stored)
+            const bool upper = wk.rows > BM / 2;
             for (int kb = 0; kb < nkb; ++kb) {
                 if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, p.err, p.wait_limit_ns)) { ok = false; break; }
                 inflight &= ~(1u << stage);
-                mbar_expect_tx(&full[stage], 2 * A_BYTES + B_BYTES);
+                mbar_expect_tx(&full[stage], (upper ? 2 * A_BYTES : A_BYTES) + B_BYTES);
                 tma_load_2d(sA1 + stage * A_BYTES, &tm_a1, kb * BK, (int)wk.row0, &full[stage]);
                 tma_load_2d(sA2 + stage * A_BYTES, &tm_a2, kb * BK, (int)wk.row0, &full[stage]);
+                if (upper) {
+                    tma_load_2d(sA1 + stage * A_BYTES + A_BYTES / 2, &tm_a1, kb * BK, (int)wk.row0 + BM / 2, &full[stage]);
+                    tma_load_2d(sA2 + stage * A_BYTES + A_BYTES / 2, &tm_a2, kb * BK, (int)wk.row0 + BM / 2, &full[stage]);
+                }
                 tma_load_2d(sB + stage * B_BYTES, &tm_b0, kb * BK, b0, &full[stage]);
                 tma_load_2d(sB + stage * B_BYTES + B_BYTES / 2, &tm_b1, kb * BK, b1, &full[stage]);
                 inflight |= 1u << stage;
@@ -308,40 +317,37 @@ tc_fp8_gemm_kernel(const __grid_constant__ CUtensorMap tm_a1, const __grid_const
         const int c1 = p.swiglu ? BN / 2 + 64 * half : 128 * half + 64;
         uint32_t kbg = 0;
         for (int w = blockIdx.x; w < total; w += gridDim.x) {
-            const Work wk = decode_work(p, w);
-            const int64_t row = wk.row0 + r;
-            const bool in_range = row < p.n_rows;
-            // scales: the activation row's, and the weight n-blocks of this thread's columns
-            const float* sa = p.a_scale + (in_range ? row : 0) * kq;
-            const float* s0;
-            const float* s1;
-            if (p.swiglu) {  // 128 gate rows nt*128..: n-block nt of the gate scales; up the same
-                s0 = p.w_scale0 + ((int64_t)wk.e * nb_per_e + wk.nt) * kq;
-                s1 = p.w_scale1 + ((int64_t)wk.e * nb_per_e + wk.nt) * kq;
-            } else {  // down columns 128*half ..: n-block 2*nt + half
-                s0 = p.w_scale0 + ((int64_t)wk.e * nb_per_e + 2 * wk.nt + half) * kq;
-                s1 = s0;
+            // scales: the activation row's, and the weight n-blocks of this
+            // thread's columns, as element offsets (int: the scale tensors
+            // hold far fewer than 2^31 entries)
+            int sa_off, s_off;
+            {
+                const Work wk = decode_work(p, w);
+                const int64_t row = wk.row0 + r;
+                sa_off = row < p.n_rows ? (int)(row * kq) : -1;
+                // gate/up: 128 gate rows nt*128.. are n-block nt of the gate scales, up the same;
+                // down: columns 128*half .. are n-block 2*nt + half
+                s_off = (wk.e * nb_per_e + (p.swiglu ? wk.nt : 2 * wk.nt + half)) * kq;
             }
             float acc[128];
 #pragma unroll
             for (int i = 0; i < 128; ++i) acc[i] = 0.0f;
-            // the k block's scales, loaded two k blocks ahead so that the
-            // promotion never waits on a global load
+            // the k block's scales, loaded one k block ahead (a k block of
+            // MMAs takes far longer than a load) so that the promotion does
+            // not wait on them
             auto scales_of = [&](int kb, float& a, float& w0, float& w1) {
                 const bool ok_kb = kb < nkb;
-                a = in_range && ok_kb ? sa[kb] : 0.0f;
-                w0 = ok_kb ? s0[kb] : 0.0f;
-                w1 = ok_kb ? s1[kb] : 0.0f;
+                a = sa_off >= 0 && ok_kb ? p.a_scale[sa_off + kb] : 0.0f;
+                w0 = ok_kb ? p.w_scale0[s_off + kb] : 0.0f;
+                w1 = ok_kb ? p.w_scale1[s_off + kb] : 0.0f;  // the same block of the up (or down) scales
             };
-            float a0, x0, y0, a1, x1, y1;
+            float a0, x0, y0;
             scales_of(0, a0, x0, y0);
-            scales_of(1, a1, x1, y1);
             bool ok = true;
             for (int kb = 0; kb < nkb; ++kb, ++kbg) {
                 const uint32_t pb = kbg & 1u, pph = (kbg >> 1) & 1u;
                 const float f0 = a0 * x0, f1 = a0 * y0;
-                a0 = a1; x0 = x1; y0 = y1;
-                scales_of(kb + 2, a1, x1, y1);
+                scales_of(kb + 1, a0, x0, y0);
                 if (!warp_wait(&pfull[pb], pph, abort_flag, p.err, p.wait_limit_ns)) { ok = false; break; }
                 tc_fence_after();
                 const uint32_t tb = t_row + pb * BN;
@@ -359,6 +365,8 @@ tc_fp8_gemm_kernel(const __grid_constant__ CUtensorMap tm_a1, const __grid_const
                 if (lane == 0) mbar_arrive(&pempty[pb]);
             }
             if (!ok) break;
+            const Work wk = decode_work(p, w);
+            const int64_t row = wk.row0 + r;
             if (r < wk.rows) {
                 if (p.swiglu) {
                     __nv_bfloat16* dst = p.out + row * (int64_t)p.out_cols + wk.nt * (BN / 2) + 64 * half;
@@ -453,10 +461,10 @@ cudaError_t launch_ffn_tc_fp8(const FfnProblem& p, cudaStream_t stream) {
     const uint8_t* aq = static_cast<const uint8_t*>(p.a_q);
     const uint8_t* hq = static_cast<const uint8_t*>(p.h_q);
     CUtensorMap ma1, ma2, mg, mu, mh1, mh2, md;
-    if (!map_e4m3(&ma1, aq, p.n_rows, p.H, BM) || !map_e4m3(&ma2, aq + p.n_rows * p.H, p.n_rows, p.H, BM) ||
+    if (!map_e4m3(&ma1, aq, p.n_rows, p.H, BM / 2) || !map_e4m3(&ma2, aq + p.n_rows * p.H, p.n_rows, p.H, BM / 2) ||
         !map_e4m3(&mg, p.w_gate, (int64_t)p.E * p.I, p.H, BN / 2) ||
-        !map_e4m3(&mu, p.w_up, (int64_t)p.E * p.I, p.H, BN / 2) || !map_e4m3(&mh1, hq, p.n_rows, p.I, BM) ||
-        !map_e4m3(&mh2, hq + p.n_rows * p.I, p.n_rows, p.I, BM) ||
+        !map_e4m3(&mu, p.w_up, (int64_t)p.E * p.I, p.H, BN / 2) || !map_e4m3(&mh1, hq, p.n_rows, p.I, BM / 2) ||
+        !map_e4m3(&mh2, hq + p.n_rows * p.I, p.n_rows, p.I, BM / 2) ||
         !map_e4m3(&md, p.w_down, (int64_t)p.E * p.H, p.I, BN / 2))
         return cudaErrorInvalidValue;
     Params g{};
