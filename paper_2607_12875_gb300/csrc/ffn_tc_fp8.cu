@@ -82,7 +82,6 @@ struct Params {
     int n_tiles;            // N tiles per M tile
     int out_cols;           // row length of the output
     int b_rows_per_expert;  // rows of the B tensor per expert
-    int swiglu;             // 1: gate/up GEMM with SwiGLU epilogue; 0: plain output
     const int32_t* counts;
     const int32_t* offsets;
     const int32_t* sched;
@@ -117,9 +116,10 @@ __device__ __forceinline__ Work decode_work(const Params& p, int w) {
 }
 
 // first B row (in the stacked [E * rows_per_expert, K] tensor) of each tile half
+template <bool SWIGLU>
 __device__ __forceinline__ void b_rows(const Params& p, const Work& wk, int& b0, int& b1) {
-    b0 = wk.e * p.b_rows_per_expert + (p.swiglu ? wk.nt * (BN / 2) : wk.nt * BN);
-    b1 = p.swiglu ? b0 : b0 + BN / 2;
+    b0 = wk.e * p.b_rows_per_expert + (SWIGLU ? wk.nt * (BN / 2) : wk.nt * BN);
+    b1 = SWIGLU ? b0 : b0 + BN / 2;
 }
 
 // ---------------------------------------------- activation quantisation
@@ -191,6 +191,7 @@ quant_rows_kernel(const __nv_bfloat16* __restrict__ src, const int32_t* __restri
 
 // -------------------------------------------------------------- the GEMM
 
+template <bool SWIGLU>  // gate/up GEMM with the SwiGLU epilogue, or the down GEMM
 __global__ void __launch_bounds__(THREADS, 1)
 tc_fp8_gemm_kernel(const __grid_constant__ CUtensorMap tm_a1, const __grid_constant__ CUtensorMap tm_a2,
                    const __grid_constant__ CUtensorMap tm_b0, const __grid_constant__ CUtensorMap tm_b1,
@@ -247,7 +248,7 @@ tc_fp8_gemm_kernel(const __grid_constant__ CUtensorMap tm_a1, const __grid_const
         for (int w = blockIdx.x; w < total && ok; w += gridDim.x) {
             const Work wk = decode_work(p, w);
             int b0, b1;
-            b_rows(p, wk, b0, b1);
+            b_rows<SWIGLU>(p, wk, b0, b1);
             // A in two 64-row boxes; the second only when the tile has rows
             // there (the MMA's rows past the tile's end read whatever the slot
             // held, and their accumulators are never stored)
@@ -313,8 +314,8 @@ tc_fp8_gemm_kernel(const __grid_constant__ CUtensorMap tm_a1, const __grid_const
         const int kq = p.K / QB;
         const int nb_per_e = p.b_rows_per_expert / QB;
         // this thread's 128 columns: 64 gate + the matching 64 up (SwiGLU), or 128 down
-        const int c0 = p.swiglu ? 64 * half : 128 * half;
-        const int c1 = p.swiglu ? BN / 2 + 64 * half : 128 * half + 64;
+        const int c0 = SWIGLU ? 64 * half : 128 * half;
+        const int c1 = SWIGLU ? BN / 2 + 64 * half : 128 * half + 64;
         uint32_t kbg = 0;
         for (int w = blockIdx.x; w < total; w += gridDim.x) {
             // scales: the activation row's, and the weight n-blocks of this
@@ -327,7 +328,7 @@ tc_fp8_gemm_kernel(const __grid_constant__ CUtensorMap tm_a1, const __grid_const
                 sa_off = row < p.n_rows ? (int)(row * kq) : -1;
                 // gate/up: 128 gate rows nt*128.. are n-block nt of the gate scales, up the same;
                 // down: columns 128*half .. are n-block 2*nt + half
-                s_off = (wk.e * nb_per_e + (p.swiglu ? wk.nt : 2 * wk.nt + half)) * kq;
+                s_off = (wk.e * nb_per_e + (SWIGLU ? wk.nt : 2 * wk.nt + half)) * kq;
             }
             float acc[128];
 #pragma unroll
@@ -368,7 +369,7 @@ tc_fp8_gemm_kernel(const __grid_constant__ CUtensorMap tm_a1, const __grid_const
             const Work wk = decode_work(p, w);
             const int64_t row = wk.row0 + r;
             if (r < wk.rows) {
-                if (p.swiglu) {
+                if constexpr (SWIGLU) {
                     __nv_bfloat16* dst = p.out + row * (int64_t)p.out_cols + wk.nt * (BN / 2) + 64 * half;
 #pragma unroll
                     for (int c = 0; c < 8; ++c) {
@@ -426,16 +427,18 @@ static cudaError_t launch_quant(const void* src, const int32_t* sorted_pair, int
     return cudaGetLastError();
 }
 
+template <bool SWIGLU>
 static cudaError_t launch_gemm(const CUtensorMap& a1, const CUtensorMap& a2, const CUtensorMap& b0,
                                const CUtensorMap& b1, const Params& prm, int64_t max_work, cudaStream_t stream) {
     static DeviceOnce smem_set;
     cudaError_t e = smem_set.run([] {
-        return cudaFuncSetAttribute(tc_fp8_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+        return cudaFuncSetAttribute(tc_fp8_gemm_kernel<SWIGLU>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    SMEM_BYTES);
     });
     if (e != cudaSuccess) return e;
     const int grid = (int)min64(sm_count(), max_work);
     if (grid <= 0) return cudaSuccess;
-    if (const cudaError_t le = launch_k(tc_fp8_gemm_kernel, dim3(grid), dim3(THREADS), SMEM_BYTES, stream, a1, a2,
+    if (const cudaError_t le = launch_k(tc_fp8_gemm_kernel<SWIGLU>, dim3(grid), dim3(THREADS), SMEM_BYTES, stream, a1, a2,
                                         b0, b1, prm);
         le != cudaSuccess)
         return le;
@@ -468,21 +471,21 @@ cudaError_t launch_ffn_tc_fp8(const FfnProblem& p, cudaStream_t stream) {
         !map_e4m3(&md, p.w_down, (int64_t)p.E * p.H, p.I, BN / 2))
         return cudaErrorInvalidValue;
     Params g{};
-    g.K = p.H; g.n_tiles = p.I / (BN / 2); g.out_cols = p.I; g.b_rows_per_expert = p.I; g.swiglu = 1;
+    g.K = p.H; g.n_tiles = p.I / (BN / 2); g.out_cols = p.I; g.b_rows_per_expert = p.I;
     g.counts = p.counts; g.offsets = p.offsets; g.sched = p.sched; g.E = p.E; g.n_rows = p.n_rows;
     g.out = static_cast<__nv_bfloat16*>(p.h); g.err = p.err;
     g.a_scale = p.a_s;
     g.w_scale0 = static_cast<const float*>(p.s_gate); g.w_scale1 = static_cast<const float*>(p.s_up);
     g.wait_limit_ns = tc_wait_limit_ns();
-    if ((err = launch_gemm(ma1, ma2, mg, mu, g, max_m * g.n_tiles, stream)) != cudaSuccess) return err;
+    if ((err = launch_gemm<true>(ma1, ma2, mg, mu, g, max_m * g.n_tiles, stream)) != cudaSuccess) return err;
     // h quantised per 1x128 for the down GEMM
     if ((err = launch_quant(p.h, nullptr, 1, p.n_rows, p.I, p.h_q, p.h_s, stream)) != cudaSuccess) return err;
     Params d = g;
-    d.K = p.I; d.n_tiles = p.H / BN; d.out_cols = p.H; d.b_rows_per_expert = p.H; d.swiglu = 0;
+    d.K = p.I; d.n_tiles = p.H / BN; d.out_cols = p.H; d.b_rows_per_expert = p.H;
     d.out = static_cast<__nv_bfloat16*>(p.y);
     d.a_scale = p.h_s;
     d.w_scale0 = static_cast<const float*>(p.s_down); d.w_scale1 = d.w_scale0;
-    return launch_gemm(mh1, mh2, md, md, d, max_m * d.n_tiles, stream);
+    return launch_gemm<false>(mh1, mh2, md, md, d, max_m * d.n_tiles, stream);
 }
 
 }  // namespace gbmoe
