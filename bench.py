@@ -57,7 +57,7 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 TRAFFIC_PER_ACTIVE_EXPERT: dict = {
     ("decode_bf16_T32_H4096_E128_k8_I1536", "stream"): 1.0966e9 / 29,
     ("prefill_bf16_T8192_H4096_E128_k8_I1536", "tc"): 1.6655e9 / 32,
-    ("dsv3_fp8_T2048_H7168_E256s1_k8_I2048", "tc_fp8"): 3.0185e9 / 64,
+    ("dsv3_fp8_T2048_H7168_E256s1_k8_I2048", "tc_fp8"): 2.9962e9 / 64,
     ("dsv4_mxfp4_T2048_H7168_E256s1_k8_I2048", "tc"): 1.6565e9 / 64,
 }
 
