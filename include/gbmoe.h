@@ -28,6 +28,11 @@
  *  - Calls that take a workspace use it for scratch only; its size comes from
  *    gbmoe_workspace_size for the same config. Calls sharing one workspace
  *    must not overlap in time (same stream, or ordered by events).
+ *  - The library keeps per-device state for the life of the process (kernel
+ *    shared-memory limits set once, SM counts, occupancy, the static
+ *    scratch of moe_permute_noalloc). A reset of a device's context
+ *    (cudaDeviceReset) discards what the driver held of it: make no further
+ *    call on that device in the same process.
  *  - Names: T tokens, H hidden size, E routed experts, k = top_k, I expert
  *    intermediate size, P = T*k (token, slot) pairs, pair p = t*k + j.
  */
@@ -328,8 +333,11 @@ int moe_device_status(void* workspace, void* stream, int32_t* status);
  * return GBMOE_EUNSUPPORTED without launching anything. The call allocates
  * nothing. Its first call on each device looks up the array's device
  * address (cudaGetSymbolAddress, with that device current), so make that
- * first call before any stream capture. All calls share the array: calls
- * that overlap on the GPU (unordered streams) race; order them.
+ * first call before any stream capture. The looked-up address is kept for
+ * the life of the process and does not survive a reset of the device's
+ * context (cudaDeviceReset): do not call this after one. All calls share
+ * the array: calls that overlap on the GPU (unordered streams) race; order
+ * them.
  */
 int moe_permute_noalloc(const gbmoe_config* cfg, const int32_t* topk_ids, int32_t* counts, int32_t* offsets,
                         int32_t* sorted_pair, int32_t* pair_pos, void* stream);

@@ -12,6 +12,9 @@
 // device address. Its device address is looked up once per device, with
 // that device current, by cudaGetSymbolAddress; the first call on each
 // device does this and should therefore come before any stream capture.
+// The address is kept until the process exits: a reset of the device's
+// context (cudaDeviceReset) would leave it stale, so the call is not for
+// processes that reset a device and go on.
 // All calls share the array and it keeps the previous call's contents, so
 // two calls that overlap on the GPU (different streams, no ordering) race.
 // The scan and scatter overwrite every entry they read, so nothing needs
