@@ -183,7 +183,9 @@ int gbmoe_last_cuda_error(void);
 
 /* GBMOE_OK if the config is valid and covered, else the status a call with it
  * would return. Limits: H % 256 == 0, I % 128 == 0 (I_shared too),
- * 1 <= E <= 512, 1 <= top_k <= min(E, 32), T >= 0, P <= 2^30. */
+ * 1 <= E <= 512, 1 <= top_k <= min(E, 32), T >= 0, P <= 2^30; with fp8
+ * weights also P * kb < 2^31 and E * kb^2 < 2^31, kb = max(H, I, I_shared) /
+ * 128 (the fp8 route indexes its scale tensors with 32-bit offsets). */
 int gbmoe_check_config(const gbmoe_config* cfg);
 
 /* Workspace bytes that moe_forward / moe_forward_hostio need for cfg (the

@@ -1,6 +1,8 @@
 // C ABI of the MoE layer (declared in include/gbmoe.h): argument checks on
 // the host, workspace carving, and the launch sequence of the layer's nodes
 // (MoE Gate -> Fused MoE -> Weight Sum) on the caller's stream.
+#include <algorithm>
+#include <climits>
 #include <cmath>
 #include <cstdint>
 #include <cstring>
@@ -59,6 +61,13 @@ int check_cfg(const gbmoe_config* c) {
     if (bf16_gemm_route(c->ffn_route) && c->act_dtype != GBMOE_BF16) return GBMOE_EUNSUPPORTED;
     if (c->ffn_route == GBMOE_FFN_TC_FP8 && (c->act_dtype != GBMOE_BF16 || c->w_dtype != GBMOE_FP8_E4M3_B128))
         return GBMOE_EUNSUPPORTED;
+    if (c->w_dtype == GBMOE_FP8_E4M3_B128) {
+        // the fp8 route addresses its activation and weight scales with 32-bit
+        // offsets (far more rows than any device could hold the codes of)
+        const int64_t kb = std::max({c->H, c->I, c->has_shared ? c->I_shared : 0}) / 128;
+        if ((int64_t)c->T * c->top_k * kb > INT32_MAX || (int64_t)c->E * kb * kb > INT32_MAX)
+            return GBMOE_EUNSUPPORTED;
+    }
     return GBMOE_OK;
 }
 

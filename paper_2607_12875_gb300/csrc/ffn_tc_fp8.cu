@@ -319,8 +319,8 @@ tc_fp8_gemm_kernel(const __grid_constant__ CUtensorMap tm_a1, const __grid_const
         uint32_t kbg = 0;
         for (int w = blockIdx.x; w < total; w += gridDim.x) {
             // scales: the activation row's, and the weight n-blocks of this
-            // thread's columns, as element offsets (int: the scale tensors
-            // hold far fewer than 2^31 entries)
+            // thread's columns, as element offsets (int: the library refuses
+            // fp8 configs whose scale tensors reach 2^31 entries)
             int sa_off, s_off;
             {
                 const Work wk = decode_work(p, w);

@@ -84,6 +84,20 @@ def test_invalid_configs_are_rejected(lib, change, status):
     assert gb.workspace_size(c) == 0
 
 
+def test_fp8_configs_keep_scale_offsets_in_32_bits(lib):
+    """The fp8 route indexes its scale tensors with 32-bit offsets: a batch
+    whose activation scales would reach 2^31 entries is refused (P * H/128 >=
+    2^31 at H = 7168 from P = 38.35 M pairs), one just below passes."""
+    kb = synth.WORKLOADS[4].H // 128
+    limit_pairs = (2 ** 31 - 1) // kb
+    below = cfg_of(4, T=limit_pairs // 8)
+    above = cfg_of(4, T=limit_pairs // 8 + 1)
+    assert below.T * 8 * kb <= 2 ** 31 - 1 < above.T * 8 * kb
+    assert gb.check_config(below) == gb.OK
+    assert gb.check_config(above) == gb.EUNSUPPORTED
+    assert gb.check_config(cfg_of(1, T=limit_pairs)) == gb.OK  # fp32 weights: no such limit
+
+
 def test_sigmoid_group_rules(lib):
     c = cfg_of(4)
     for ch in (dict(n_group=7), dict(topk_group=9), dict(top_k=200, topk_group=1)):
