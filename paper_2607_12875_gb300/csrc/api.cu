@@ -312,6 +312,33 @@ FfnProblem shared_problem(const gbmoe_config* c, const void* x, const gbmoe_expe
     return p;
 }
 
+// Every host-side check of moe_forward (x and out: the device buffers the
+// layer reads and writes), so that a caller can run them before it enqueues
+// anything of its own.
+int check_forward(const gbmoe_config* cfg, const void* x, const void* w_router, const float* logit_bias,
+                  const float* select_bias, const gbmoe_expert_weights* experts, const gbmoe_expert_weights* shared,
+                  const void* out, const int32_t* topk_ids, const float* topk_w, const int32_t* counts_out, void* ws,
+                  size_t ws_bytes) {
+    int s = check_cfg(cfg);
+    if (s) return s;
+    if (cfg->T == 0) return check_ws(cfg, ws, ws_bytes);  // nothing to read or write
+    if (!x || !w_router || !out || !aligned(x, 16) || !aligned(w_router, 16) || !aligned(out, 16))
+        return GBMOE_EINVAL;
+    if ((logit_bias && !aligned(logit_bias, 4)) || (select_bias && !aligned(select_bias, 4))) return GBMOE_EINVAL;
+    if ((topk_ids && !aligned(topk_ids, 4)) || (topk_w && !aligned(topk_w, 4)) ||
+        (counts_out && !aligned(counts_out, 4)))
+        return GBMOE_EINVAL;
+    if ((s = check_weights(cfg, experts))) return s;
+    if (cfg->has_shared && (s = check_weights(cfg, shared))) return s;
+    if ((s = check_ws(cfg, ws, ws_bytes))) return s;
+    // every route must be launchable before anything is enqueued: the routed
+    // problem with I, the shared one with I_shared
+    if ((s = route_launchable(cfg, pick_route(cfg, (int64_t)cfg->T * cfg->top_k, cfg->E, cfg->I), cfg->I))) return s;
+    if (cfg->has_shared && (s = route_launchable(cfg, pick_route(cfg, cfg->T, 1, cfg->I_shared), cfg->I_shared)))
+        return s;
+    return GBMOE_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -441,27 +468,14 @@ int moe_forward(const gbmoe_config* cfg, const void* x, const void* w_router, co
                 const float* select_bias, const gbmoe_expert_weights* experts, const gbmoe_expert_weights* shared,
                 void* out, int32_t* topk_ids, float* topk_w, int32_t* counts_out, void* ws, size_t ws_bytes,
                 void* stream) {
-    int s = check_cfg(cfg);
-    if (s) return s;
-    if (cfg->T == 0) return check_ws(cfg, ws, ws_bytes);  // nothing to read or write
-    if (!x || !w_router || !out || !aligned(x, 16) || !aligned(w_router, 16) || !aligned(out, 16))
-        return GBMOE_EINVAL;
-    if ((logit_bias && !aligned(logit_bias, 4)) || (select_bias && !aligned(select_bias, 4))) return GBMOE_EINVAL;
-    if ((topk_ids && !aligned(topk_ids, 4)) || (topk_w && !aligned(topk_w, 4)) ||
-        (counts_out && !aligned(counts_out, 4)))
-        return GBMOE_EINVAL;
-    if ((s = check_weights(cfg, experts))) return s;
-    if (cfg->has_shared && (s = check_weights(cfg, shared))) return s;
-    if ((s = check_ws(cfg, ws, ws_bytes))) return s;
+    int s = check_forward(cfg, x, w_router, logit_bias, select_bias, experts, shared, out, topk_ids, topk_w,
+                          counts_out, ws, ws_bytes);
+    if (s || cfg->T == 0) return s;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     const Layout L = layout(cfg);
     const int64_t P = (int64_t)cfg->T * cfg->top_k;
-    // every route must be launchable before anything is enqueued: the routed
-    // problem with I, the shared one with I_shared
     const int r_routed = pick_route(cfg, P, cfg->E, cfg->I);
-    if ((s = route_launchable(cfg, r_routed, cfg->I))) return s;
     const int r_shared = cfg->has_shared ? pick_route(cfg, cfg->T, 1, cfg->I_shared) : GBMOE_FFN_SIMT;
-    if (cfg->has_shared && (s = route_launchable(cfg, r_shared, cfg->I_shared))) return s;
     if (const cudaError_t ce = cudaMemsetAsync(at<int32_t>(ws, L.err), 0, 4, st); ce != cudaSuccess) return cuda_status(ce);
     int32_t* ids = at<int32_t>(ws, L.ids);
     float* w = at<float>(ws, L.w);
@@ -519,6 +533,10 @@ int moe_forward_hostio(const gbmoe_config* cfg, const void* x_host, const void* 
     const size_t bytes = (size_t)cfg->T * cfg->H * act_bytes(cfg->act_dtype);
     void* xin = at<char>(ws, L.xin);
     void* xout = at<char>(ws, L.xout);
+    // the layer's own checks first, so that a bad argument enqueues no copy
+    if ((s = check_forward(cfg, xin, w_router, logit_bias, select_bias, experts, shared, xout, nullptr, nullptr,
+                           nullptr, ws, ws_bytes)))
+        return s;
     if (bytes && (s = cuda_status(cudaMemcpyAsync(xin, x_host, bytes, cudaMemcpyHostToDevice, st)))) return s;
     s = moe_forward(cfg, xin, w_router, logit_bias, select_bias, experts, shared, xout, nullptr, nullptr, nullptr, ws,
                     ws_bytes, stream);

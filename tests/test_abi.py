@@ -230,3 +230,25 @@ def test_sorted_copy_of_x_only_where_a_gemm_reads_it(lib):
     dq = gb.workspace_size(cfg_of(5, ffn_route=gb.FFN_TC_DEQUANT))         # bf16 copy, then gathers
     weights_copy = 3 * w5.E * w5.H * w5.I * 2
     assert dq - in_gemm == pytest.approx(weights_copy - w5.P * w5.H * 2, abs=512)
+
+
+def test_hostio_checks_the_layer_arguments_before_copying(lib):
+    """moe_forward_hostio runs moe_forward's own checks (router weights,
+    expert weights, scales, routes) before it enqueues the host-to-device
+    copy of x: a bad argument returns with nothing enqueued."""
+    c = cfg_of(1)
+    x_host, out_host, p = FakePtr(), FakePtr(), FakePtr()
+    ws = FakePtr(gb.workspace_size(c))
+    w = gb.weights(p, p, p)
+    with pytest.raises(gb.GbmoeError) as e:
+        gb.moe_forward_hostio(c, x_host, None, None, None, w, None, out_host, ws, stream=0)  # no router weights
+    assert e.value.status == gb.EINVAL
+    with pytest.raises(gb.GbmoeError) as e:
+        gb.moe_forward_hostio(c, x_host, p, None, None, gb.weights(p, None, p), None, out_host, ws, stream=0)
+    assert e.value.status == gb.EINVAL
+    c4 = cfg_of(4, T=16)  # fp8 weights without their scales
+    ws4 = FakePtr(gb.workspace_size(c4))
+    with pytest.raises(gb.GbmoeError) as e:
+        gb.moe_forward_hostio(c4, x_host, p, None, None, gb.weights(p, p, p), gb.weights(p, p, p), out_host, ws4,
+                              stream=0)
+    assert e.value.status == gb.EINVAL
