@@ -449,7 +449,7 @@ def measure(args, wid: int, overrides, dist, world: int, rank: int, local: int, 
 
 
 # workloads the default run times besides the headline one: prefill bf16,
-# DeepSeek-style fp8 and skewed int4 (the benchmark spec's other size classes),
+# DeepSeek-style fp8 and skewed int4 (the other size classes of the layer),
 # and the DeepSeek-style layer with MXFP4 experts
 PER_CONFIG = (3, 4, 5, 6)
 
