@@ -1013,7 +1013,7 @@ cudaError_t launch_ffn_tc(const FfnProblem& pin, cudaStream_t stream) {
         if (!p.x_sorted) return cudaErrorInvalidValue;  // the workspace holds no sorted copy for this route
         const int vpr = p.H * 2 / 16;
         const int64_t nvec = p.n_rows * vpr;
-        const int gblocks = (int)min64((nvec + 255) / 256, 152 * 16);
+        const int gblocks = (int)min64((nvec + 255) / 256, (int64_t)sm_count() * 16);
         if (const cudaError_t le = launch_k(gather_rows_kernel, dim3(gblocks), dim3(256), 0, stream,
                 static_cast<const uint4*>(p.x), p.sorted_pair, p.pair_div, p.n_rows, vpr,
                 static_cast<uint4*>(p.x_sorted)); le != cudaSuccess)
