@@ -100,7 +100,8 @@ enum {
     GBMOE_FFN_TC_FP8 = 5,     /* fp8 tensor cores: FP8_E4M3_B128 weights as stored,
                                  activations quantised to e4m3 per 1x128 block      */
     GBMOE_FFN_TC_PAIR = 6,    /* as TC on CTA pairs: one MMA of 256 rows per pair
-                                 (each CTA holds and decodes half the weight tile)  */
+                                 (each CTA holds half the weight tile); bf16
+                                 weights only (quantised: TC_PAIR_DEQUANT)          */
     GBMOE_FFN_TC_PAIR_DEQUANT = 7 /* as TC_DEQUANT, the bf16 GEMM on CTA pairs      */
 };
 
